@@ -1,0 +1,301 @@
+// C ABI entry points of libchronostitch: argument validation on the host,
+// kernel launches, and the per-device status word that kernels write when
+// they detect a data error or a bounded wait gives up.
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+
+#include "cs_device.cuh"
+#include "cs_internal.h"
+
+namespace cs {
+
+// Per-device status word (static storage of this module, one copy per device).
+__device__ unsigned int g_status[kStatusWords];
+
+namespace {
+
+thread_local char t_detail[512] = "no error";
+
+constexpr int kMaxDevices = 64;
+std::mutex g_mu;
+unsigned int *g_status_addr[kMaxDevices] = {};
+
+cudaStream_t as_stream(void *s) { return static_cast<cudaStream_t>(s); }
+
+// theta_i / (2 pi) in units of 2^-64 turns, rounded to nearest, from the fp64
+// value of theta_i = theta^(-2i/D).  theta_i = m * 2^e exactly (m < 2^53); the
+// product with round(2^66 / (2 pi)) is formed in 128-bit integer arithmetic.
+unsigned long long turn_step(double theta_i) {
+    int e;
+    const double fr = std::frexp(theta_i, &e);                    // theta_i = fr * 2^e, fr in [0.5,1)
+    const unsigned long long m = static_cast<unsigned long long>(std::ldexp(fr, 53));  // exact
+    e -= 53;                                                       // theta_i = m * 2^e
+    const unsigned __int128 inv2pi_66 = 0xa2f9836e4e44152aull;     // round(2^66 / (2 pi))
+    const unsigned __int128 prod = static_cast<unsigned __int128>(m) * inv2pi_66;
+    // step = prod * 2^(e - 2); theta_i <= 1 gives e <= -53, a right shift of >= 55
+    const int sh = 2 - e;
+    if (sh >= 128) return 0;
+    const unsigned __int128 half = static_cast<unsigned __int128>(1) << (sh - 1);
+    return static_cast<unsigned long long>((prod + half) >> sh);
+}
+
+}  // namespace
+
+cs_status fail(cs_status s, const char *fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    std::vsnprintf(t_detail, sizeof(t_detail), fmt, ap);
+    va_end(ap);
+    return s;
+}
+
+cs_status cuda_fail(cudaError_t e, const char *what) {
+    return fail(CS_ERR_CUDA, "%s: %s (%s)", what, cudaGetErrorName(e), cudaGetErrorString(e));
+}
+
+unsigned int *status_word() {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) {
+        cuda_fail(e, "cudaGetDevice");
+        return nullptr;
+    }
+    if (dev < 0 || dev >= kMaxDevices) {
+        fail(CS_ERR_UNSUPPORTED, "device ordinal %d beyond %d", dev, kMaxDevices);
+        return nullptr;
+    }
+    std::lock_guard<std::mutex> lock(g_mu);
+    if (g_status_addr[dev] == nullptr) {
+        void *p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_status);
+        if (e != cudaSuccess) {
+            cuda_fail(e, "cudaGetSymbolAddress(status word)");
+            return nullptr;
+        }
+        g_status_addr[dev] = static_cast<unsigned int *>(p);
+    }
+    return g_status_addr[dev];
+}
+
+}  // namespace cs
+
+using namespace cs;
+
+extern "C" {
+
+int cs_abi_version(void) { return 1; }
+
+const char *cs_status_string(cs_status s) {
+    switch (s) {
+        case CS_OK: return "ok";
+        case CS_ERR_INVALID_ARG: return "invalid argument";
+        case CS_ERR_UNSUPPORTED: return "unsupported configuration";
+        case CS_ERR_CUDA: return "CUDA error";
+        case CS_ERR_TIMEOUT: return "device wait timed out";
+        case CS_ERR_DEVICE_ARG: return "device data check failed";
+    }
+    return "unknown status";
+}
+
+const char *cs_last_error_detail(void) { return t_detail; }
+
+cs_status cs_rebase_keys(const void *k_in, void *k_out, cs_dtype dtype, int n_layers,
+                         int64_t layer_stride, int T, int n_kv_heads, int head_dim,
+                         const int32_t *pos_local, const int32_t *pos_global,
+                         const cs_rope_cfg *rope, void *stream) {
+    if (dtype != CS_DTYPE_F32 && dtype != CS_DTYPE_BF16) return fail(CS_ERR_INVALID_ARG, "dtype");
+    if (n_layers < 0 || T < 0 || n_kv_heads <= 0 || head_dim <= 0)
+        return fail(CS_ERR_INVALID_ARG, "negative size or non-positive head count/dim");
+    if (head_dim != 128) return fail(CS_ERR_UNSUPPORTED, "head_dim %d (only 128)", head_dim);
+    const int max_heads = dtype == CS_DTYPE_BF16 ? 32 : 16;
+    if (n_kv_heads > max_heads)
+        return fail(CS_ERR_UNSUPPORTED, "n_kv_heads %d > %d", n_kv_heads, max_heads);
+    if (rope == nullptr) return fail(CS_ERR_INVALID_ARG, "rope config is NULL");
+    if (!(std::isfinite(rope->theta) && rope->theta > 1.0))
+        return fail(CS_ERR_INVALID_ARG, "rope theta must be finite and > 1");
+    long long ssum = 0;
+    for (int a = 0; a < 3; ++a) {
+        if (rope->sections[a] < 0) return fail(CS_ERR_INVALID_ARG, "negative mrope section");
+        ssum += rope->sections[a];
+    }
+    if (ssum != head_dim / 2)
+        return fail(CS_ERR_INVALID_ARG, "mrope sections sum to %lld, need %d", ssum, head_dim / 2);
+    const long long row = static_cast<long long>(n_kv_heads) * head_dim;
+    if (layer_stride < static_cast<long long>(T) * row)
+        return fail(CS_ERR_INVALID_ARG, "layer_stride %lld < T*n_kv_heads*head_dim",
+                    static_cast<long long>(layer_stride));
+    if (n_layers == 0 || T == 0) return CS_OK;
+    if (k_in == nullptr || k_out == nullptr || pos_local == nullptr || pos_global == nullptr)
+        return fail(CS_ERR_INVALID_ARG, "NULL tensor pointer");
+    if (!aligned16(k_in) || !aligned16(k_out) || (layer_stride * (dtype == CS_DTYPE_BF16 ? 2 : 4)) % 16)
+        return fail(CS_ERR_INVALID_ARG, "keys must be 16-byte aligned (pointers and layer stride)");
+    if (k_in != k_out) {
+        const long long esz = dtype == CS_DTYPE_BF16 ? 2 : 4;
+        const long long span = ((n_layers - 1) * layer_stride + T * row) * esz;
+        const char *a = static_cast<const char *>(k_in);
+        const char *b = static_cast<const char *>(k_out);
+        if (a < b + span && b < a + span)
+            return fail(CS_ERR_INVALID_ARG, "k_in and k_out overlap without being equal");
+    }
+    RebaseArgs args;
+    std::memset(&args, 0, sizeof(args));
+    args.k_in = k_in;
+    args.k_out = k_out;
+    args.n_layers = n_layers;
+    args.layer_stride = layer_stride;
+    args.T = T;
+    args.hkv = n_kv_heads;
+    args.pos_local = pos_local;
+    args.pos_global = pos_global;
+    args.in_place = (k_in == k_out);
+    int i = 0;
+    for (int a = 0; a < 3; ++a)
+        for (int c = 0; c < rope->sections[a]; ++c, ++i) args.axis[i] = static_cast<unsigned char>(a);
+    for (i = 0; i < head_dim / 2; ++i)
+        args.turn_step[i] = turn_step(std::pow(rope->theta, -(2.0 * i) / head_dim));
+    const cudaError_t e = launch_rebase(args, dtype, as_stream(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "rebase launch");
+    return CS_OK;
+}
+
+cs_status cs_score_deviation(const void *k_fresh, const void *k_cached, cs_dtype dtype, int n,
+                             int n_kv_heads, int head_dim, int64_t fresh_row_stride,
+                             int64_t cached_row_stride, float *score_out, void *stream) {
+    if (dtype != CS_DTYPE_F32 && dtype != CS_DTYPE_BF16) return fail(CS_ERR_INVALID_ARG, "dtype");
+    if (n < 0 || n_kv_heads <= 0 || head_dim <= 0)
+        return fail(CS_ERR_INVALID_ARG, "negative size or non-positive head count/dim");
+    if (head_dim != 128) return fail(CS_ERR_UNSUPPORTED, "head_dim %d (only 128)", head_dim);
+    const long long E = static_cast<long long>(n_kv_heads) * head_dim;
+    if (E > 2048) return fail(CS_ERR_UNSUPPORTED, "row of %lld elements > 2048", E);
+    if (fresh_row_stride < E || cached_row_stride < E)
+        return fail(CS_ERR_INVALID_ARG, "row stride shorter than n_kv_heads*head_dim");
+    if (n == 0) return CS_OK;
+    if (k_fresh == nullptr || k_cached == nullptr || score_out == nullptr)
+        return fail(CS_ERR_INVALID_ARG, "NULL pointer");
+    const long long esz = dtype == CS_DTYPE_BF16 ? 2 : 4;
+    if (!aligned16(k_fresh) || !aligned16(k_cached) || (fresh_row_stride * esz) % 16 ||
+        (cached_row_stride * esz) % 16)
+        return fail(CS_ERR_INVALID_ARG, "rows must start 16-byte aligned");
+    const cudaError_t e = launch_score(k_fresh, k_cached, dtype, n, static_cast<int>(E),
+                                       fresh_row_stride, cached_row_stride, score_out,
+                                       as_stream(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "score launch");
+    return CS_OK;
+}
+
+cs_status cs_select_topk(const float *score, int n, int k, int32_t idx_base, int32_t *out_idx,
+                         void *stream) {
+    if (n < 0 || k < 0 || k > n) return fail(CS_ERR_INVALID_ARG, "need 0 <= k <= n (n=%d k=%d)", n, k);
+    if (idx_base < 0 || static_cast<long long>(idx_base) + n > 0x7FFFFFFFll)
+        return fail(CS_ERR_INVALID_ARG, "idx_base + n must stay within int32");
+    if (k == 0) return CS_OK;
+    if (score == nullptr || out_idx == nullptr) return fail(CS_ERR_INVALID_ARG, "NULL pointer");
+    const cudaError_t e = launch_select(score, n, k, idx_base, out_idx, as_stream(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "select launch");
+    return CS_OK;
+}
+
+cs_status cs_repair_attention(const void *q, const void *k, const void *v, void *o, float *lse,
+                              cs_dtype dtype, int n_layers, int M, int T, int n_q_heads,
+                              int n_kv_heads, int head_dim, int64_t kv_layer_stride,
+                              const int32_t *qpos, float scale, void *stream) {
+    if (dtype != CS_DTYPE_F32 && dtype != CS_DTYPE_BF16) return fail(CS_ERR_INVALID_ARG, "dtype");
+    if (n_layers < 0 || M < 0 || T < 0 || n_q_heads <= 0 || n_kv_heads <= 0 || head_dim <= 0)
+        return fail(CS_ERR_INVALID_ARG, "negative size or non-positive head count/dim");
+    if (head_dim != 128) return fail(CS_ERR_UNSUPPORTED, "head_dim %d (only 128)", head_dim);
+    if (n_q_heads % n_kv_heads)
+        return fail(CS_ERR_INVALID_ARG, "n_q_heads %d not a multiple of n_kv_heads %d", n_q_heads,
+                    n_kv_heads);
+    if (n_q_heads / n_kv_heads > 128)
+        return fail(CS_ERR_UNSUPPORTED, "more than 128 query heads per kv head");
+    if (!std::isfinite(scale)) return fail(CS_ERR_INVALID_ARG, "scale must be finite");
+    if (kv_layer_stride < static_cast<long long>(T) * n_kv_heads * head_dim)
+        return fail(CS_ERR_INVALID_ARG, "kv_layer_stride < T*n_kv_heads*head_dim");
+    if (n_layers == 0 || M == 0) return CS_OK;
+    if (T == 0) return fail(CS_ERR_INVALID_ARG, "query rows need at least one key (T = 0)");
+    if (q == nullptr || k == nullptr || v == nullptr || o == nullptr || qpos == nullptr)
+        return fail(CS_ERR_INVALID_ARG, "NULL pointer");
+    const long long esz = dtype == CS_DTYPE_BF16 ? 2 : 4;
+    if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) ||
+        (kv_layer_stride * esz) % 16)
+        return fail(CS_ERR_INVALID_ARG, "q, k, v, o must be 16-byte aligned (and the layer stride)");
+    if (dtype == CS_DTYPE_BF16 && static_cast<long long>(M) * n_q_heads > 0x7FFFFFFFll)
+        return fail(CS_ERR_UNSUPPORTED, "M * n_q_heads too large");
+    unsigned int *status = status_word();
+    if (status == nullptr) return CS_ERR_CUDA;
+    AttnArgs a;
+    a.q = q;
+    a.k = k;
+    a.v = v;
+    a.o = o;
+    a.lse = lse;
+    a.n_layers = n_layers;
+    a.M = M;
+    a.T = T;
+    a.hq = n_q_heads;
+    a.hkv = n_kv_heads;
+    a.kv_layer_stride = kv_layer_stride;
+    a.qpos = qpos;
+    a.scale = scale;
+    a.status = status;
+    if (dtype == CS_DTYPE_F32) {
+        const cudaError_t e = launch_attn_f32(a, as_stream(stream));
+        if (e != cudaSuccess) return cuda_fail(e, "attention launch");
+        return CS_OK;
+    }
+    return launch_attn_tc(a, as_stream(stream));
+}
+
+cs_status cs_sync_status(void *stream) {
+    cudaError_t e = cudaStreamSynchronize(as_stream(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+    unsigned int *status = status_word();
+    if (status == nullptr) return CS_ERR_CUDA;
+    unsigned int host[kStatusWords] = {0, 0, 0, 0};
+    e = cudaMemcpy(host, status, sizeof(host), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(e, "reading the status word");
+    if (host[0] == 0) return CS_OK;
+    const unsigned int zero[kStatusWords] = {0, 0, 0, 0};
+    e = cudaMemcpy(status, zero, sizeof(zero), cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return cuda_fail(e, "clearing the status word");
+    const cs_status s = host[0] == 4u ? CS_ERR_TIMEOUT : CS_ERR_DEVICE_ARG;
+    return fail(s, "device status %u at site %u (detail %u)", host[0], host[1], host[2]);
+}
+
+}  // extern "C"
+
+// ---- diagnostics: a bounded wait that nothing completes -----------------------
+namespace cs {
+namespace {
+__global__ void wait_timeout_kernel(unsigned int *status, unsigned long long limit_ns) {
+    __shared__ uint64_t bar;
+    __shared__ int abort;
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        abort = 0;
+        fence_mbar_init();
+    }
+    __syncthreads();
+    // phase 0 never completes: nobody arrives on the barrier
+    mbar_wait_bounded(&bar, 0, &abort, status, kSiteDebugWait, limit_ns);
+}
+}  // namespace
+
+cudaError_t launch_wait_timeout(unsigned int *status, unsigned int limit_us, cudaStream_t s) {
+    wait_timeout_kernel<<<1, 1, 0, s>>>(status, 1000ull * limit_us);
+    return cudaGetLastError();
+}
+}  // namespace cs
+
+extern "C" cs_status cs_debug_wait_timeout(uint32_t limit_us, void *stream) {
+    if (limit_us == 0 || limit_us > 10u * 1000u * 1000u)
+        return fail(CS_ERR_INVALID_ARG, "limit_us must be in (0, 10 s]");
+    unsigned int *status = status_word();
+    if (status == nullptr) return CS_ERR_CUDA;
+    const cudaError_t e = launch_wait_timeout(status, limit_us, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "wait-timeout launch");
+    return CS_OK;
+}

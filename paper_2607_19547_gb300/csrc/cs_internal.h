@@ -1,0 +1,71 @@
+// Host-side declarations shared by the translation units of libchronostitch.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/chronostitch.h"
+
+namespace cs {
+
+// Device status word layout (one per device, zeroed by cs_sync_status):
+//   word[0]  first error code recorded (CS_ERR_TIMEOUT / CS_ERR_DEVICE_ARG), 0 if none
+//   word[1]  where it happened (kernel-specific site tag)
+//   word[2]  extra detail (block index, row, ...)
+constexpr int kStatusWords = 4;
+
+// Returns the device address of the status word of the current device, or
+// nullptr on a CUDA error (the detail is recorded for cs_last_error_detail).
+unsigned int *status_word();
+
+// Records a detail string for cs_last_error_detail and returns `s`.
+cs_status fail(cs_status s, const char *fmt, ...);
+cs_status cuda_fail(cudaError_t e, const char *what);
+
+inline bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// ---- re-base (rebase.cu) ---------------------------------------------------
+struct RebaseArgs {
+    const void *k_in;
+    void *k_out;
+    int n_layers;
+    long long layer_stride;
+    int T;
+    int hkv;
+    const int *pos_local;
+    const int *pos_global;
+    unsigned long long turn_step[64];   // theta_i / (2 pi) in units of 2^-64 turns
+    unsigned char axis[64];             // sigma(i)
+    int in_place;
+};
+cudaError_t launch_rebase(const RebaseArgs &a, cs_dtype dt, cudaStream_t s);
+
+// ---- score (score.cu) --------------------------------------------------------
+cudaError_t launch_score(const void *fresh, const void *cached, cs_dtype dt, int n, int E,
+                         long long fresh_stride, long long cached_stride, float *out,
+                         cudaStream_t s);
+
+// ---- select (select.cu) ------------------------------------------------------
+cudaError_t launch_select(const float *score, int n, int k, int idx_base, int *out,
+                          cudaStream_t s);
+
+// ---- attention (attn_f32.cu, attn_tc.cu) -------------------------------------
+struct AttnArgs {
+    const void *q;
+    const void *k;
+    const void *v;
+    void *o;
+    float *lse;
+    int n_layers, M, T, hq, hkv;
+    long long kv_layer_stride;
+    const int *qpos;
+    float scale;
+    unsigned int *status;
+};
+cudaError_t launch_attn_f32(const AttnArgs &a, cudaStream_t s);
+// Returns CS_OK, or an error status with the detail recorded.
+cs_status launch_attn_tc(const AttnArgs &a, cudaStream_t s);
+
+cudaError_t launch_wait_timeout(unsigned int *status, unsigned int limit_us, cudaStream_t s);
+
+}  // namespace cs

@@ -17,3 +17,13 @@ def golden():
     import json
     with open(os.path.join(ROOT, "tests", "golden", "paper_figures.json")) as f:
         return json.load(f)
+
+
+@pytest.fixture(scope="session")
+def cslib():
+    """The CUDA library, built in-tree if needed (nvcc cross-compiles without a GPU)."""
+    from paper_2607_19547_gb300 import _build
+    _build.build()
+    import paper_2607_19547_gb300 as cs
+    cs.lib()
+    return cs

@@ -1,0 +1,148 @@
+"""The C ABI without a GPU: every declared entry point is exported, and host-side
+argument checks reject bad calls before any CUDA work (so they run on a CPU machine)."""
+import ctypes
+import os
+import re
+import subprocess
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "chronostitch.h")
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(cs_[a-z_0-9]+)\s*\(", text)))
+
+
+def test_header_declares_the_four_steps():
+    names = declared_functions()
+    for n in ("cs_rebase_keys", "cs_score_deviation", "cs_select_topk", "cs_repair_attention",
+              "cs_sync_status", "cs_status_string"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(cslib):
+    out = subprocess.run(["nm", "-D", "--defined-only", cslib.LIB_PATH], capture_output=True,
+                         text=True, check=True).stdout
+    exported = set(re.findall(r"\s[TW]\s+(\S+)", out))
+    missing = [n for n in declared_functions() if n not in exported]
+    assert not missing, missing
+    handle = ctypes.CDLL(cslib.LIB_PATH)
+    for n in declared_functions():
+        assert getattr(handle, n) is not None
+
+
+def test_status_strings(cslib):
+    L = cslib.lib()
+    assert cslib.cs_abi_version() == 1
+    for code in range(6):
+        assert L.cs_status_string(code)
+    assert cslib.cs_status_string(0) == "ok"
+    assert "timed out" in cslib.cs_status_string(4)
+
+
+def _rope(theta=1e6, sec=(16, 24, 24)):
+    import paper_2607_19547_gb300 as cs
+    return cs._RopeCfg(theta, (ctypes.c_int32 * 3)(*sec))
+
+
+FAKE = 1 << 20   # aligned non-null address: never dereferenced when validation fails
+
+
+def test_rebase_rejects_bad_arguments(cslib):
+    L = cslib.lib()
+    r = _rope()
+
+    def call(**kw):
+        a = dict(k_in=FAKE, k_out=FAKE, dt=1, L=2, stride=4 * 2 * 128, T=4, H=2, D=128,
+                 pl=FAKE, pg=FAKE, rope=ctypes.byref(r))
+        a.update(kw)
+        return L.cs_rebase_keys(a["k_in"], a["k_out"], a["dt"], a["L"], a["stride"], a["T"],
+                                a["H"], a["D"], a["pl"], a["pg"], a["rope"], None)
+
+    assert call(D=64) == cslib.CS_ERR_UNSUPPORTED
+    assert "head_dim" in cslib.cs_last_error_detail()
+    assert call(dt=7) == cslib.CS_ERR_INVALID_ARG
+    assert call(T=-1) == cslib.CS_ERR_INVALID_ARG
+    assert call(stride=100) == cslib.CS_ERR_INVALID_ARG
+    bad = _rope(sec=(16, 24, 23))
+    assert call(rope=ctypes.byref(bad)) == cslib.CS_ERR_INVALID_ARG
+    assert "sections" in cslib.cs_last_error_detail()
+    neg = _rope(sec=(-8, 48, 24))
+    assert call(rope=ctypes.byref(neg)) == cslib.CS_ERR_INVALID_ARG
+    low = _rope(theta=1.0)
+    assert call(rope=ctypes.byref(low)) == cslib.CS_ERR_INVALID_ARG
+    assert call(rope=None) == cslib.CS_ERR_INVALID_ARG
+    assert call(k_in=None) == cslib.CS_ERR_INVALID_ARG
+    assert call(k_in=FAKE + 8, k_out=FAKE + 8) == cslib.CS_ERR_INVALID_ARG     # misaligned
+    assert call(k_out=FAKE + 256) == cslib.CS_ERR_INVALID_ARG                  # partial overlap
+    assert call(H=40) == cslib.CS_ERR_UNSUPPORTED
+    # nothing to do: succeeds without touching the device
+    assert call(L=0, k_in=None, k_out=None) == cslib.CS_OK
+    assert call(T=0, k_in=None, k_out=None, stride=0) == cslib.CS_OK
+
+
+def test_score_rejects_bad_arguments(cslib):
+    L = cslib.lib()
+
+    def call(**kw):
+        a = dict(f=FAKE, c=FAKE, dt=1, n=5, H=2, D=128, fs=256, cs=256, out=FAKE)
+        a.update(kw)
+        return L.cs_score_deviation(a["f"], a["c"], a["dt"], a["n"], a["H"], a["D"], a["fs"],
+                                    a["cs"], a["out"], None)
+
+    assert call(D=96) == cslib.CS_ERR_UNSUPPORTED
+    assert call(fs=128) == cslib.CS_ERR_INVALID_ARG
+    assert call(out=None) == cslib.CS_ERR_INVALID_ARG
+    assert call(fs=260) == cslib.CS_ERR_INVALID_ARG         # 520-byte rows break 16 B alignment
+    assert call(H=17) == cslib.CS_ERR_UNSUPPORTED
+    assert call(n=0, f=None, c=None, out=None) == cslib.CS_OK
+
+
+def test_select_rejects_bad_arguments(cslib):
+    L = cslib.lib()
+    assert L.cs_select_topk(FAKE, 10, 11, 0, FAKE, None) == cslib.CS_ERR_INVALID_ARG
+    assert L.cs_select_topk(FAKE, 10, -1, 0, FAKE, None) == cslib.CS_ERR_INVALID_ARG
+    assert L.cs_select_topk(FAKE, 10, 3, 0x7FFFFFFF - 5, FAKE, None) == cslib.CS_ERR_INVALID_ARG
+    assert L.cs_select_topk(FAKE, 10, 3, -1, FAKE, None) == cslib.CS_ERR_INVALID_ARG
+    assert L.cs_select_topk(None, 10, 3, 0, FAKE, None) == cslib.CS_ERR_INVALID_ARG
+    assert L.cs_select_topk(None, 10, 0, 0, None, None) == cslib.CS_OK
+
+
+def test_attention_rejects_bad_arguments(cslib):
+    L = cslib.lib()
+
+    def call(**kw):
+        a = dict(q=FAKE, k=FAKE, v=FAKE, o=FAKE, lse=None, dt=1, L=2, M=3, T=10, Hq=16, Hkv=2,
+                 D=128, st=10 * 2 * 128, qpos=FAKE, scale=0.0884)
+        a.update(kw)
+        return L.cs_repair_attention(a["q"], a["k"], a["v"], a["o"], a["lse"], a["dt"], a["L"],
+                                     a["M"], a["T"], a["Hq"], a["Hkv"], a["D"], a["st"],
+                                     a["qpos"], a["scale"], None)
+
+    assert call(Hq=15) == cslib.CS_ERR_INVALID_ARG
+    assert call(D=64) == cslib.CS_ERR_UNSUPPORTED
+    assert call(st=100) == cslib.CS_ERR_INVALID_ARG
+    assert call(scale=float("nan")) == cslib.CS_ERR_INVALID_ARG
+    assert call(T=0, st=0) == cslib.CS_ERR_INVALID_ARG
+    assert call(qpos=None) == cslib.CS_ERR_INVALID_ARG
+    assert call(o=FAKE + 4) == cslib.CS_ERR_INVALID_ARG
+    assert call(Hq=256, Hkv=1) == cslib.CS_ERR_UNSUPPORTED
+    assert call(M=0, q=None, o=None) == cslib.CS_OK
+
+
+def test_debug_wait_rejects_bad_limits(cslib):
+    L = cslib.lib()
+    assert L.cs_debug_wait_timeout(0, None) == cslib.CS_ERR_INVALID_ARG
+    assert L.cs_debug_wait_timeout(20_000_000, None) == cslib.CS_ERR_INVALID_ARG
+
+
+def test_python_binding_refuses_cpu_tensors(cslib):
+    import torch
+    k = torch.zeros(1, 4, 2, 128, dtype=torch.bfloat16)
+    pos = torch.zeros(4, 3, dtype=torch.int32)
+    with pytest.raises(ValueError):
+        cslib.cs_rebase_keys(k, pos, pos)

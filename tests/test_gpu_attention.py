@@ -1,0 +1,132 @@
+"""Repair attention (Eq. 1 over selected rows, causal in global order) on the GPU
+against the fp64 oracle: max-abs 2e-2 for bf16 outputs, 1e-5 for fp32."""
+import numpy as np
+import pytest
+import torch
+
+import cs_workloads as W
+import oracle as O
+from _helpers import TOL, cuda, f64
+
+pytestmark = pytest.mark.gpu
+
+
+def _rand(shape, seed, dtype):
+    g = torch.Generator(device="cuda").manual_seed(seed)
+    return torch.randn(shape, generator=g, device="cuda").to(dtype)
+
+
+def _run_and_check(cs, q, k, v, qpos, name, rows=None, layers=None, check_lse=True):
+    L, M, Hq, D = q.shape
+    lse = torch.full((L, M, Hq), float("nan"), dtype=torch.float32, device="cuda")
+    out = cs.cs_repair_attention(q, k, v, cuda(qpos), lse=lse)
+    cs.cs_sync_status()
+    rows = np.arange(M) if rows is None else np.asarray(rows)
+    layers = np.arange(L) if layers is None else np.asarray(layers)
+    qq = f64(q[torch.as_tensor(layers, device="cuda")][:, torch.as_tensor(rows, device="cuda")])
+    kk = f64(k[torch.as_tensor(layers, device="cuda")])
+    vv = f64(v[torch.as_tensor(layers, device="cuda")])
+    eo, el = O.repair_attention(qq, kk, vv, np.asarray(qpos)[rows])
+    go = f64(out[torch.as_tensor(layers, device="cuda")][:, torch.as_tensor(rows, device="cuda")])
+    err = np.max(np.abs(go - eo))
+    assert err <= TOL[name], f"max abs error {err}"
+    if check_lse:
+        gl = lse[torch.as_tensor(layers, device="cuda")][:, torch.as_tensor(rows, device="cuda")]
+        np.testing.assert_allclose(gl.cpu().numpy(), el, atol=1e-3 if name == "bf16" else 1e-5)
+    return err
+
+
+def test_tiny_f32_config_full(cslib):
+    w = W.CONFIGS["tiny_f32"]
+    x = W.make_inputs(w, seed=0, device="cuda")
+    rng = np.random.default_rng(0)
+    qpos = np.sort(rng.choice(np.arange(w.cand0, w.T), size=w.M, replace=False)).astype(np.int32)
+    _run_and_check(cslib, x["q"], x["k"], x["v"], qpos, "f32")
+
+
+@pytest.mark.parametrize("Hq,Hkv", [(16, 2), (28, 4), (2, 1), (8, 8), (7, 1), (32, 2)])
+def test_bf16_group_sizes_ragged(cslib, Hq, Hkv):
+    L, T, M = 2, 1000, 37
+    q = _rand((L, M, Hq, 128), 1, torch.bfloat16)
+    k = _rand((L, T, Hkv, 128), 2, torch.bfloat16)
+    v = _rand((L, T, Hkv, 128), 3, torch.bfloat16)
+    rng = np.random.default_rng(Hq)
+    qpos = np.sort(rng.choice(T, size=M, replace=False)).astype(np.int32)
+    qpos[0] = 0
+    _run_and_check(cslib, q, k, v, qpos, "bf16")
+
+
+def test_bf16_dense_rows_and_block_edges(cslib):
+    """Consecutive rows and rows on key-block boundaries (127, 128, 255, 256, ...)."""
+    L, T, Hq, Hkv = 1, 700, 16, 2
+    q = _rand((L, 40, Hq, 128), 4, torch.bfloat16)
+    k = _rand((L, T, Hkv, 128), 5, torch.bfloat16)
+    v = _rand((L, T, Hkv, 128), 6, torch.bfloat16)
+    qpos = np.array(sorted(set(list(range(0, 20)) + [126, 127, 128, 129, 254, 255, 256, 257,
+                                                        383, 384, 511, 512, 513, 639, 640,
+                                                        698, 699])), np.int32)[:40]
+    q = q[:, :len(qpos)].contiguous()
+    _run_and_check(cslib, q, k, v, qpos, "bf16")
+
+
+def test_bf16_large_logits_rescale(cslib):
+    """Keys growing along the sequence force the running maximum to rise block after block."""
+    L, T, Hq, Hkv = 1, 1024, 8, 1
+    q = _rand((L, 16, Hq, 128), 7, torch.float32)
+    k = _rand((L, T, Hkv, 128), 8, torch.float32) * torch.linspace(0.1, 4.0, T,
+                                                                   device="cuda")[None, :, None, None]
+    v = _rand((L, T, Hkv, 128), 9, torch.float32)
+    qpos = np.linspace(100, T - 1, 16).astype(np.int32)
+    _run_and_check(cslib, (q * 2).to(torch.bfloat16), k.to(torch.bfloat16),
+                   v.to(torch.bfloat16), qpos, "bf16")
+
+
+def test_qwen3b_4x1024_all_rows(cslib):
+    w = W.CONFIGS["qwen3b_4x1024"]
+    x = W.make_inputs(w, seed=0, device="cuda")
+    rng = np.random.default_rng(1)
+    qpos = np.sort(rng.choice(np.arange(w.cand0, w.cand0 + w.n_cand), size=w.M,
+                              replace=False)).astype(np.int32)
+    _run_and_check(cslib, x["q"], x["k"], x["v"], qpos, "bf16", layers=[0, 1, 17, 35])
+
+
+@pytest.mark.parametrize("name", ["qwen3b_16x1024_q64", "qwen3b_64x1024_r30", "qwen7b_32x2048"])
+def test_large_configs_sampled_rows(cslib, name):
+    w = W.CONFIGS[name]
+    x = W.make_inputs(w, seed=0, device="cuda")
+    rng = np.random.default_rng(2)
+    sel = np.sort(rng.choice(np.arange(w.cand0, w.cand0 + w.n_cand), size=w.k, replace=False))
+    qpos = np.concatenate([sel, np.arange(w.T - w.suffix, w.T)]).astype(np.int32)
+    rows = W.sample_rows(w.M, 48, seed=5)
+    _run_and_check(cslib, x["q"], x["k"], x["v"], qpos, "bf16", rows=rows,
+                   layers=[0, w.n_layers - 1])
+
+
+def test_single_key_and_empty(cslib):
+    q = _rand((1, 1, 16, 128), 10, torch.bfloat16)
+    k = _rand((1, 5, 2, 128), 11, torch.bfloat16)
+    v = _rand((1, 5, 2, 128), 12, torch.bfloat16)
+    out = cslib.cs_repair_attention(q, k, v, cuda(np.array([0], np.int32)))
+    cslib.cs_sync_status()
+    # one visible key: every head of group g returns v[0, 0, g]
+    for h in range(16):
+        assert torch.allclose(out[0, 0, h].float(), v[0, 0, h // 8].float(), atol=1e-2)
+    empty = cslib.cs_repair_attention(q[:, :0].contiguous(), k, v,
+                                      cuda(np.zeros(0, np.int32)))
+    cslib.cs_sync_status()
+    assert empty.numel() == 0
+
+
+def test_bad_query_positions_are_reported(cslib):
+    q = _rand((1, 4, 16, 128), 13, torch.bfloat16)
+    k = _rand((1, 64, 2, 128), 14, torch.bfloat16)
+    bad = cuda(np.array([3, 10, 70, 20], np.int32))       # out of range and not ascending
+    cslib.cs_repair_attention(q, k, k, bad)
+    with pytest.raises(cslib.CsError) as e:
+        cslib.cs_sync_status()
+    assert e.value.status == cslib.CS_ERR_DEVICE_ARG
+    cslib.cs_sync_status()                                 # cleared after reporting
+    q32, k32 = q.float(), k.float()
+    cslib.cs_repair_attention(q32, k32, k32, bad)
+    with pytest.raises(cslib.CsError):
+        cslib.cs_sync_status()

@@ -1,0 +1,95 @@
+"""Score (Eq. 5) and top-rho selection (Sec. 2) on the GPU against the oracle.
+
+The score that the selection ranks is defined in one fixed fp32 order, so GPU
+and oracle must agree bit for bit; indices must agree exactly."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from _helpers import cuda, f64
+
+pytestmark = pytest.mark.gpu
+
+
+def _rows(n, H, dtype, seed, scale=1.0):
+    g = torch.Generator(device="cuda").manual_seed(seed)
+    return (torch.randn((n, H, 128), generator=g, device="cuda") * scale).to(dtype)
+
+
+@pytest.mark.parametrize("H", [1, 2, 4, 7, 8])
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+@pytest.mark.parametrize("n", [1, 37, 3072])
+def test_score_bit_exact(cslib, H, dtype, n):
+    a = _rows(n, H, dtype, 1 + H + n)
+    b = (a.float() + _rows(n, H, torch.float32, 7 + H + n) *
+         torch.exp(_rows(n, 1, torch.float32, 9)[:, :, :1])).to(dtype)
+    got = cslib.cs_score_deviation(a, b)
+    cslib.cs_sync_status()
+    exp = O.score_f32_canonical(f64(a).astype(np.float32), f64(b).astype(np.float32))
+    assert np.array_equal(got.cpu().numpy().view(np.uint32), exp.view(np.uint32))
+    np.testing.assert_allclose(got.cpu().numpy(), O.score_f64(f64(a), f64(b)), rtol=2e-6)
+
+
+def test_score_strided_rows_and_exact_cases(cslib):
+    # rows taken from a [L, T, H, D] cache slice: stride H*D, plus a padded fresh buffer
+    cache = _rows(4 * 50, 2, torch.bfloat16, 3).view(4, 50, 2, 128)
+    cached = cache[1, 10:40]
+    fresh_buf = torch.zeros((30, 3, 128), dtype=torch.bfloat16, device="cuda")
+    fresh_buf[:, :2] = _rows(30, 2, torch.bfloat16, 4)
+    fresh = fresh_buf[:, :2]
+    got = cslib.cs_score_deviation(fresh, cached)
+    cslib.cs_sync_status()
+    exp = O.score_f32_canonical(f64(fresh).astype(np.float32), f64(cached).astype(np.float32))
+    assert np.array_equal(got.cpu().numpy().view(np.uint32), exp.view(np.uint32))
+    same = cslib.cs_score_deviation(cached.contiguous(), cached)
+    cslib.cs_sync_status()
+    assert torch.count_nonzero(same).item() == 0
+    # worked by hand: ((1 + 2^-24) + (2^-24 + 2^-24)) = 1 + 2^-23 in the fixed order
+    a = torch.zeros((1, 2, 128), dtype=torch.float32, device="cuda")
+    a[0, 0, :4] = torch.tensor([1.0, 2 ** -12, 2 ** -12, 2 ** -12])
+    z = cslib.cs_score_deviation(a, torch.zeros_like(a))
+    cslib.cs_sync_status()
+    assert z.item() == np.float32(1.0 + 2.0 ** -23)
+
+
+def _check_select(cs, vals, k, base):
+    s = cuda(np.asarray(vals, np.float32))
+    got = cs.cs_select_topk(s, k, base)
+    cs.cs_sync_status()
+    exp = O.select_topk(np.asarray(vals, np.float32), k, base)
+    assert np.array_equal(got.cpu().numpy(), exp)
+
+
+@pytest.mark.parametrize("n", [1, 7, 1023, 1024, 1025, 3072, 64512, 100003])
+def test_select_matches_oracle(cslib, n):
+    rng = np.random.default_rng(n)
+    cont = (rng.lognormal(0, 1.5, n) * 256).astype(np.float32)
+    ties = rng.choice(np.array([0, 1, 2, 3.5, 1e30], np.float32), n)
+    for vals in (cont, ties):
+        for k in sorted({0, 1, n // 7, n // 2, max(n - 1, 0), n}):
+            _check_select(cslib, vals, k, 1032)
+
+
+def test_select_special_values(cslib):
+    vals = np.array([1.0, np.inf, np.nan, 0.0, -1.0, 3.0, -0.0, -np.inf, 3.0, np.inf],
+                    np.float32)
+    for k in range(len(vals) + 1):
+        _check_select(cslib, vals, k, 0)
+    eq = np.full(5000, 2.5, np.float32)
+    _check_select(cslib, eq, 1234, 17)        # all equal: lowest indices
+
+
+def test_select_fraction_of_candidates(cslib):
+    """k = ceil(rho * N_c) of the candidates with idx_base at the first candidate."""
+    rng = np.random.default_rng(0)
+    n_cand, cand0 = 3072, 1032
+    vals = (rng.lognormal(0, 1, n_cand) * 256).astype(np.float32)
+    k = O.k_from_rho(1500, n_cand)
+    s = cuda(vals)
+    got = cslib.cs_select_topk(s, k, cand0).cpu().numpy()
+    cslib.cs_sync_status()
+    assert len(got) == 461 and got[0] >= cand0 and got[-1] < cand0 + n_cand
+    assert np.all(np.diff(got) > 0)
+    kth = np.sort(vals)[::-1][k - 1]
+    assert np.all(vals[got - cand0] >= kth)
