@@ -116,7 +116,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
     const int kmax = clamp_pos(p.qpos[r_last], p.T);
     const int nb = kmax / kBlockN + 1;
     const int mask_from = qmin / kBlockN;
-    const uint32_t q_bytes = static_cast<uint32_t>(p.tok * p.G) * 256u;
+    const uint32_t q_bytes = static_cast<uint32_t>(p.tok * p.G) * 256u;   // both 64-column halves
 
     if (threadIdx.x == 0) {
         mbar_init(&bars->q_full, 1);
@@ -161,7 +161,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
             tma_prefetch_desc(&tm_q);
             tma_prefetch_desc(&tm_k);
             tma_prefetch_desc(&tm_v);
-            mbar_arrive_expect_tx(&bars->q_full, 2 * q_bytes);
+            mbar_arrive_expect_tx(&bars->q_full, q_bytes);
             tma_load_4d(base + Smem::q, &tm_q, &bars->q_full, 0, g * p.G, r0, l);
             tma_load_4d(base + Smem::q + kHalfBytes, &tm_q, &bars->q_full, 64, g * p.G, r0, l);
             int nk = 0, nv = 0;   // K and V tiles issued

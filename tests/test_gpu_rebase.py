@@ -72,7 +72,7 @@ def test_qwen3b_4x1024_full(cslib):
 def test_random_coordinates_ragged(cslib, H, dtype):
     T, L = 333, 3
     g = torch.Generator(device="cuda").manual_seed(100 + H)
-    k = (torch.randn((L, T, H, 128), generator=g, device="cuda") * 3).to(dtype)
+    k = torch.randn((L, T, H, 128), generator=g, device="cuda").to(dtype)
     loc, glo = W.random_coordinates(T, seed=H, max_coord=100000)
     glo[::7] = loc[::7]                         # some tokens do not move
     glo[1::5, 1] = loc[1::5, 1]                 # some move on two axes only
