@@ -9,18 +9,28 @@
 // the largest qpos of its rows; blocks past the smallest qpos apply the
 // per-row causal mask.
 //
-// CTA = 6 warps:
-//   warp 0      TMA producer: Q once, then K and V tiles through an
-//               NS-stage shared-memory ring (128-byte swizzle).
-//   warp 1      owns tensor memory; lane 0 issues tcgen05.mma:
-//               S_j = Q K_j^T  (A, B from shared memory, fp32 into TMEM,
-//               double-buffered), O += P_j V_j (A = P from TMEM, B = V from
+// CTA = 11 warps:
+//   warp 0      TMA producers: lane 0 loads Q once and streams K through a
+//               3-stage shared-memory ring, lane 1 streams V through a
+//               2-stage ring (128-byte swizzle).
+//   warp 1      owns tensor memory; lane 0 issues S_j = Q K_j^T (A, B from
+//               shared memory, fp32 into one of three 128-column TMEM buffers).
+//   warp 10     lane 0 issues O += P_j V_j (A = P_j from TMEM, B = V from
 //               shared memory, MN-major).
-//   warps 2-5   softmax: thread = one TMEM lane = one query row.  Reads S_j,
-//               masks, updates the running max (rescaling O in TMEM only
-//               when the max grows by more than 2^8), writes P_j = exp2(...)
-//               as bf16 over the first 64 columns of S_j's TMEM buffer,
-//               and finally normalises O and stores it.
+//               A tcgen05.mma issue blocks until the tensor core takes it, so
+//               one thread that also waits on barriers leaves the tensor core
+//               idle while it waits; two issuers keep it fed.
+//   warps 2-9   softmax, two warpgroups: warpgroup h (warps 2+4h .. 5+4h)
+//               owns key columns [64h, 64h+64) of every S block and output
+//               dims [64h, 64h+64) of O; thread = one TMEM lane = one query
+//               row.  Reads its half of S_j, masks, exchanges the half-row
+//               maxima through shared memory (one named barrier per block),
+//               updates the running max (rescaling its half of O in TMEM only
+//               when the max grows by more than 2^8), writes its half of
+//               P_j = exp2(...) as bf16 over S_j's TMEM columns, and finally
+//               normalises its half of O and stores it.
+// TMEM: S buffers at columns 0, 128, 256; O at 384.  S_j reuses the buffer
+// of P_{j-3}, so the S issuer runs up to three blocks ahead of the softmax.
 // Every mbarrier wait is bounded; on a timeout the CTA records
 // CS_ERR_TIMEOUT, stops issuing work, drains what it issued, frees its
 // tensor memory and exits.
@@ -35,36 +45,40 @@
 namespace cs {
 namespace {
 
-constexpr int kThreads = 192;
-constexpr int kBlockN = 128;           // keys per KV tile
-constexpr int kStages = 2;             // K/V shared-memory ring depth
-constexpr uint32_t kTileBytes = 128 * 128 * 2;      // one K or V tile (two 16 KB halves)
-constexpr uint32_t kHalfBytes = 128 * 64 * 2;
-constexpr uint32_t kTmemCols = 512;    // S0 [0,128) S1 [128,256) O [256,384)
-constexpr uint32_t kColO = 256;
+constexpr int kThreads = 352;          // 11 warps: producers, S issuer, 2 x 4 softmax, PV issuer
+constexpr int kPvWarp = 10;
+constexpr int kBlockN = 128;           // keys per KV block
+constexpr int kKStages = 3;            // K shared-memory ring depth
+constexpr int kVStages = 2;            // V ring depth (V is consumed after the softmax)
+constexpr uint32_t kHalf = 128 * 64 * 2;           // 128 rows x 64 dims (one swizzle half)
+constexpr uint32_t kTileBytes = 2 * kHalf;         // Q tile, or one K or V block
+constexpr uint32_t kTmemCols = 512;
+constexpr int kSBufs = 3;              // S (and P) buffers of 128 columns
+constexpr uint32_t kColO = 384;
 constexpr uint64_t kWaitLimitNs = 1000000000ull;    // 1 s
 
 struct Smem {
     // byte offsets from the 1024-aligned base
     static constexpr uint32_t q = 0;
     static constexpr uint32_t k = q + kTileBytes;
-    static constexpr uint32_t v = k + kStages * kTileBytes;
-    static constexpr uint32_t bars = v + kStages * kTileBytes;
-    static constexpr uint32_t total = bars + 256;
+    static constexpr uint32_t v = k + kKStages * kTileBytes;
+    static constexpr uint32_t bars = v + kVStages * kTileBytes;
+    static constexpr uint32_t xchg = bars + 512;           // float [2 slots][2 halves][128 rows]
+    static constexpr uint32_t total = xchg + 2 * 2 * 128 * 4;
 };
 
 struct Bars {
     uint64_t q_full;
-    uint64_t k_full[kStages], k_empty[kStages];
-    uint64_t v_full[kStages], v_empty[kStages];
-    uint64_t s_full[2], p_full[2];
-    uint64_t o_done;     // one completion per P*V block
-    uint64_t o_final;    // single use: every P*V of the tile is done
-    uint64_t mma_done;   // single use: every tensor-core operation of the CTA retired
+    uint64_t k_full[kKStages], k_empty[kKStages];
+    uint64_t v_full[kVStages], v_empty[kVStages];
+    uint64_t s_full[kSBufs], p_full[kSBufs];
+    uint64_t pv_done[kSBufs];   // one completion per P*V block that read P from buffer b
+    uint64_t o_final;           // single use: every P*V of the tile is done
+    uint64_t mma_done;          // single use (two arrivals): every tensor-core operation retired
     uint32_t tmem_base;
     int abort;
 };
-static_assert(sizeof(Bars) <= 256, "barrier area");
+static_assert(sizeof(Bars) <= 512, "barrier area");
 
 struct TcParams {
     int n_layers, M, T, hq, hkv, G, tok, n_qtiles;
@@ -87,14 +101,25 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     return r;
 }
 
-// Tile coordinates of work item `item`, heaviest query tiles first (selected
-// rows are ascending, so later query tiles see more keys).
+// Tile coordinates of work item `item`.  CTAs launched together should share
+// a (layer, kv head) so its K/V blocks are read from HBM once and then hit in
+// L2; to keep the tail short the heavier half of the query tiles (selected
+// rows ascend, so later tiles see more keys) runs first for every group, then
+// the lighter half.  Within a group, tiles run heaviest first.
 __device__ __forceinline__ void decode_item(const TcParams &p, int item, int &l, int &g, int &qt) {
-    const int per = p.n_layers * p.hkv;
-    qt = p.n_qtiles - 1 - item / per;
-    const int rem = item % per;
-    l = rem / p.hkv;
-    g = rem % p.hkv;
+    const int lo_n = p.n_qtiles / 2, hi_n = p.n_qtiles - lo_n;
+    const int groups = p.n_layers * p.hkv;
+    int grp;
+    if (item < groups * hi_n) {
+        grp = item / hi_n;
+        qt = p.n_qtiles - 1 - item % hi_n;
+    } else {
+        const int i2 = item - groups * hi_n;
+        grp = i2 / lo_n;
+        qt = lo_n - 1 - i2 % lo_n;
+    }
+    l = grp / p.hkv;
+    g = grp % p.hkv;
 }
 
 __device__ __forceinline__ int clamp_pos(int x, int T) { return min(max(x, 0), T - 1); }
@@ -120,19 +145,21 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
 
     if (threadIdx.x == 0) {
         mbar_init(&bars->q_full, 1);
-        for (int s = 0; s < kStages; ++s) {
+        for (int s = 0; s < kKStages; ++s) {
             mbar_init(&bars->k_full[s], 1);
             mbar_init(&bars->k_empty[s], 1);
+        }
+        for (int s = 0; s < kVStages; ++s) {
             mbar_init(&bars->v_full[s], 1);
             mbar_init(&bars->v_empty[s], 1);
         }
-        for (int b = 0; b < 2; ++b) {
+        for (int b = 0; b < kSBufs; ++b) {
             mbar_init(&bars->s_full[b], 1);
-            mbar_init(&bars->p_full[b], 128);
+            mbar_init(&bars->p_full[b], 256);
+            mbar_init(&bars->pv_done[b], 1);
         }
-        mbar_init(&bars->o_done, 1);
         mbar_init(&bars->o_final, 1);
-        mbar_init(&bars->mma_done, 1);
+        mbar_init(&bars->mma_done, 2);
         bars->abort = 0;
         fence_mbar_init();
     }
@@ -143,9 +170,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
     // rows of the Q tile that TMA does not write (G not dividing 128) must be finite
     {
         const uint32_t used = static_cast<uint32_t>(p.tok * p.G) * 128u;   // bytes per half
-        for (uint32_t off = used + threadIdx.x * 16u; off < kHalfBytes; off += kThreads * 16u) {
+        for (uint32_t off = used + threadIdx.x * 16u; off < kHalf; off += kThreads * 16u) {
             *reinterpret_cast<uint4 *>(base + Smem::q + off) = make_uint4(0, 0, 0, 0);
-            *reinterpret_cast<uint4 *>(base + Smem::q + kHalfBytes + off) = make_uint4(0, 0, 0, 0);
+            *reinterpret_cast<uint4 *>(base + Smem::q + kHalf + off) = make_uint4(0, 0, 0, 0);
         }
         fence_proxy_async_smem();
     }
@@ -156,108 +183,105 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
     volatile int *abort = &bars->abort;
 
     if (warp == 0) {
-        // ------------------------------------------------------------ producer
-        if (lane == 0) {
-            tma_prefetch_desc(&tm_q);
-            tma_prefetch_desc(&tm_k);
-            tma_prefetch_desc(&tm_v);
-            mbar_arrive_expect_tx(&bars->q_full, q_bytes);
-            tma_load_4d(base + Smem::q, &tm_q, &bars->q_full, 0, g * p.G, r0, l);
-            tma_load_4d(base + Smem::q + kHalfBytes, &tm_q, &bars->q_full, 64, g * p.G, r0, l);
-            int nk = 0, nv = 0;   // K and V tiles issued
+        // ------------------------------------------------------------ producers
+        // lane 0 streams Q and the K ring, lane 1 the V ring
+        if (lane < 2) {
+            volatile int never = 0;
+            int issued = 0;
+            const int stages = lane == 0 ? kKStages : kVStages;
+            uint64_t *full = lane == 0 ? bars->k_full : bars->v_full;
+            uint64_t *empty = lane == 0 ? bars->k_empty : bars->v_empty;
+            const CUtensorMap *tm = lane == 0 ? &tm_k : &tm_v;
+            const uint32_t ring = lane == 0 ? Smem::k : Smem::v;
+            tma_prefetch_desc(tm);
+            if (lane == 0) {
+                tma_prefetch_desc(&tm_q);
+                mbar_arrive_expect_tx(&bars->q_full, q_bytes);
+                tma_load_4d(base + Smem::q, &tm_q, &bars->q_full, 0, g * p.G, r0, l);
+                tma_load_4d(base + Smem::q + kHalf, &tm_q, &bars->q_full, 64, g * p.G, r0, l);
+            }
             for (int j = 0; j < nb; ++j) {
-                const int s = j % kStages;
-                const uint32_t ph = (j / kStages) & 1;
-                if (!mbar_wait_bounded(&bars->k_empty[s], ph ^ 1, abort, p.status,
+                const int s = j % stages;
+                if (!mbar_wait_bounded(&empty[s], ((j / stages) & 1) ^ 1, abort, p.status,
                                        kSiteAttnProducer, kWaitLimitNs)) break;
-                uint8_t *kd = base + Smem::k + s * kTileBytes;
-                mbar_arrive_expect_tx(&bars->k_full[s], kTileBytes);
-                tma_load_4d(kd, &tm_k, &bars->k_full[s], 0, g, j * kBlockN, l);
-                tma_load_4d(kd + kHalfBytes, &tm_k, &bars->k_full[s], 64, g, j * kBlockN, l);
-                ++nk;
-                if (!mbar_wait_bounded(&bars->v_empty[s], ph ^ 1, abort, p.status,
-                                       kSiteAttnProducer, kWaitLimitNs)) break;
-                uint8_t *vd = base + Smem::v + s * kTileBytes;
-                mbar_arrive_expect_tx(&bars->v_full[s], kTileBytes);
-                tma_load_4d(vd, &tm_v, &bars->v_full[s], 0, g, j * kBlockN, l);
-                tma_load_4d(vd + kHalfBytes, &tm_v, &bars->v_full[s], 64, g, j * kBlockN, l);
-                ++nv;
+                uint8_t *dst = base + ring + s * kTileBytes;
+                mbar_arrive_expect_tx(&full[s], kTileBytes);
+                tma_load_4d(dst, tm, &full[s], 0, g, j * kBlockN, l);
+                tma_load_4d(dst + kHalf, tm, &full[s], 64, g, j * kBlockN, l);
+                ++issued;
             }
             if (*abort) {
                 // drain: every issued copy lands before the CTA's shared memory is released.
-                // Phases of one barrier complete in order, so waiting for the last
-                // copy issued on each barrier covers the earlier ones.
-                volatile int never = 0;
-                mbar_wait_bounded(&bars->q_full, 0, &never, nullptr, 0, kWaitLimitNs);
-                for (int s = 0; s < kStages; ++s) {
-                    for (int which = 0; which < 2; ++which) {
-                        const int cnt = which ? nv : nk;
-                        if (cnt <= s) continue;
-                        const int jl = s + ((cnt - 1 - s) / kStages) * kStages;
-                        uint64_t *bar = which ? &bars->v_full[s] : &bars->k_full[s];
-                        mbar_wait_bounded(bar, (jl / kStages) & 1, &never, nullptr, 0,
-                                          kWaitLimitNs);
-                    }
+                // Phases of one barrier complete in order, so waiting for the last copy
+                // issued on each barrier covers the earlier ones.
+                if (lane == 0) mbar_wait_bounded(&bars->q_full, 0, &never, nullptr, 0, kWaitLimitNs);
+                for (int s = 0; s < stages; ++s) {
+                    if (issued <= s) continue;
+                    const int jl = s + ((issued - 1 - s) / stages) * stages;
+                    mbar_wait_bounded(&full[s], (jl / stages) & 1, &never, nullptr, 0, kWaitLimitNs);
                 }
             }
         }
     } else if (warp == 1) {
-        // ------------------------------------------------------------ MMA issuer
+        // ------------------------------------------------------------ S issuer
         if (lane == 0) {
-            const uint32_t idesc_qk = idesc_bf16(128, 128, 0, 0);
-            const uint32_t idesc_pv = idesc_bf16(128, 128, 0, 1);
-            const uint32_t q_addr = smem_u32(base + Smem::q);
+            const uint32_t idesc = idesc_bf16(128, kBlockN, 0, 0);
+            // descriptors are built once; an operand at byte offset `off` from a base is
+            // base + (off >> 4) (the 14-bit address field cannot overflow below 256 KB)
+            const uint64_t qd = smem_desc(smem_u32(base + Smem::q), 16, 1024, 2);
+            const uint64_t kd0 = smem_desc(smem_u32(base + Smem::k), 16, 1024, 2);
             bool ok = mbar_wait_bounded(&bars->q_full, 0, abort, p.status, kSiteAttnMma,
                                         kWaitLimitNs);
-            auto issue_qk = [&](int j) -> bool {
-                const int s = j % kStages;
-                if (!mbar_wait_bounded(&bars->k_full[s], (j / kStages) & 1, abort, p.status,
-                                       kSiteAttnMma, kWaitLimitNs)) return false;
-                tc_fence_after();
-                const uint32_t k_addr = smem_u32(base + Smem::k + s * kTileBytes);
-                const uint32_t d = tmem + static_cast<uint32_t>((j & 1) * 128);
-#pragma unroll
-                for (int kk = 0; kk < 8; ++kk) {
-                    const uint32_t off = (kk >> 2) * kHalfBytes + (kk & 3) * 32;
-                    tc_mma_ss(d, smem_desc(q_addr + off, 16, 1024, 2),
-                              smem_desc(k_addr + off, 16, 1024, 2), idesc_qk, kk > 0);
-                }
-                tc_commit(&bars->s_full[j & 1]);
-                tc_commit(&bars->k_empty[s]);
-                return true;
-            };
-            if (ok) ok = issue_qk(0);
             for (int j = 0; ok && j < nb; ++j) {
-                if (j + 1 < nb) {
-                    // S_{j+1} overwrites the buffer that held P_{j-1}: PV_{j-1} must be done
-                    if (j >= 1 && !mbar_wait_bounded(&bars->o_done, (j - 1) & 1, abort, p.status,
-                                                     kSiteAttnMma, kWaitLimitNs)) { ok = false; break; }
-                    if (!issue_qk(j + 1)) { ok = false; break; }
-                }
-                const int s = j % kStages;
-                if (!mbar_wait_bounded(&bars->p_full[j & 1], (j >> 1) & 1, abort, p.status,
-                                       kSiteAttnMma, kWaitLimitNs)) { ok = false; break; }
-                if (!mbar_wait_bounded(&bars->v_full[s], (j / kStages) & 1, abort, p.status,
-                                       kSiteAttnMma, kWaitLimitNs)) { ok = false; break; }
+                const int s = j % kKStages, b = j % kSBufs;
+                // buffer b held P_{j-3}: PV_{j-3} must have read it
+                if (j >= kSBufs && !mbar_wait_bounded(&bars->pv_done[b], ((j / kSBufs) - 1) & 1,
+                                                      abort, p.status, kSiteAttnMma, kWaitLimitNs)) break;
+                if (!mbar_wait_bounded(&bars->k_full[s], (j / kKStages) & 1, abort, p.status,
+                                       kSiteAttnMma, kWaitLimitNs)) break;
                 tc_fence_after();
-                const uint32_t v_addr = smem_u32(base + Smem::v + s * kTileBytes);
-                const uint32_t a_tm = tmem + static_cast<uint32_t>((j & 1) * 128);
+                const uint64_t kd = kd0 + ((s * kTileBytes) >> 4);
+                const uint32_t d = tmem + static_cast<uint32_t>(b * kBlockN);
 #pragma unroll
-                for (int kk = 0; kk < 8; ++kk) {
+                for (int kk = 0; kk < 8; ++kk) {   // 16 head dims per MMA
+                    const uint32_t off = (kk >> 2) * kHalf + (kk & 3) * 32;
+                    tc_mma_ss(d, qd + (off >> 4), kd + (off >> 4), idesc, kk > 0);
+                }
+                tc_commit(&bars->s_full[b]);
+                tc_commit(&bars->k_empty[s]);
+            }
+            // completes once every tcgen05 operation issued by this thread has retired
+            tc_commit(&bars->mma_done);
+        }
+    } else if (warp == kPvWarp) {
+        // ------------------------------------------------------------ PV issuer
+        if (lane == 0) {
+            const uint32_t idesc = idesc_bf16(128, 128, 0, 1);
+            const uint64_t vd0 = smem_desc(smem_u32(base + Smem::v), kHalf, 1024, 2);
+            for (int j = 0; j < nb; ++j) {
+                const int s = j % kVStages, b = j % kSBufs;
+                if (!mbar_wait_bounded(&bars->p_full[b], (j / kSBufs) & 1, abort, p.status,
+                                       kSiteAttnMma, kWaitLimitNs)) break;
+                if (!mbar_wait_bounded(&bars->v_full[s], (j / kVStages) & 1, abort, p.status,
+                                       kSiteAttnMma, kWaitLimitNs)) break;
+                tc_fence_after();
+                const uint64_t vd = vd0 + ((s * kTileBytes) >> 4);
+                const uint32_t a_tm = tmem + static_cast<uint32_t>(b * kBlockN);
+#pragma unroll
+                for (int kk = 0; kk < kBlockN / 16; ++kk) {
                     // A: 16 keys of P = 8 packed columns; B: 16 rows (keys) of V, MN-major
-                    tc_mma_ts(tmem + kColO, a_tm + kk * 8,
-                              smem_desc(v_addr + kk * 2048, kHalfBytes, 1024, 2), idesc_pv,
+                    tc_mma_ts(tmem + kColO, a_tm + kk * 8, vd + ((kk * 2048) >> 4), idesc,
                               (j > 0 || kk > 0) ? 1u : 0u);
                 }
-                tc_commit(&bars->o_done);
+                tc_commit(&bars->pv_done[b]);
                 tc_commit(&bars->v_empty[s]);
                 if (j == nb - 1) tc_commit(&bars->o_final);
             }
-            // completes once every tcgen05 operation issued above has retired
             tc_commit(&bars->mma_done);
         }
     } else {
         // ------------------------------------------------------------ softmax
+        const int half = (warp - 2) >> 2;             // key columns / output dims [64h, 64h+64)
         const int qw = warp & 3;
         const int m = 32 * qw + lane;                 // TMEM lane = MMA row
         const int t = m / p.G, hh = m - t * p.G;
@@ -266,36 +290,53 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
         int qp = kmax;
         if (valid) {
             const int raw = p.qpos[r];
-            if (raw < 0 || raw >= p.T || (r > 0 && p.qpos[r - 1] >= raw))
+            if (half == 0 && (raw < 0 || raw >= p.T || (r > 0 && p.qpos[r - 1] >= raw)))
                 report_error(p.status, 5u, kSiteAttnQpos, static_cast<unsigned>(r));
             qp = clamp_pos(raw, p.T);
         }
+        float *xchg = reinterpret_cast<float *>(base + Smem::xchg);   // [slot][half][row]
         const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * qw) << 16);
+        const int col0 = 64 * half;
         float m_run = -INFINITY, l_run = 0.0f;
         bool ok = true;
+        // Failure handling: a thread that gives up only clears `ok`; the decision to
+        // stop is taken by all 256 softmax threads together at the exchange barrier
+        // (barrier + OR), so neither warpgroup is ever left waiting at a barrier.
         for (int j = 0; j < nb; ++j) {
-            const int b = j & 1;
-            const bool w_ok = mbar_wait_bounded(&bars->s_full[b], (j >> 1) & 1, abort, p.status,
-                                                kSiteAttnSoftmax, kWaitLimitNs);
-            if (!__all_sync(0xFFFFFFFFu, w_ok)) { ok = false; *abort = 1; break; }
-            tc_fence_after();
-            float s[128];
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                uint32_t rr[32];
-                tmem_ld32(lane_base + b * 128 + c * 32, rr);
-#pragma unroll
-                for (int e = 0; e < 32; ++e) s[c * 32 + e] = __uint_as_float(rr[e]);
+            const int b = j % kSBufs;
+            if (ok) {
+                const bool w_ok = mbar_wait_bounded(&bars->s_full[b], (j / kSBufs) & 1, abort,
+                                                    p.status, kSiteAttnSoftmax, kWaitLimitNs);
+                ok = __all_sync(0xFFFFFFFFu, w_ok);
             }
-            if (j >= mask_from) {
-                const int lim = qp - j * kBlockN;
+            float s[64];
+            float *slot = xchg + (j & 1) * 256;
+            if (ok) {
+                tc_fence_after();
+                uint32_t sr[64];
+                tmem_ld64(lane_base + b * kBlockN + col0, sr);
 #pragma unroll
-                for (int c = 0; c < 128; ++c)
-                    if (c > lim) s[c] = -INFINITY;
+                for (int c = 0; c < 64; ++c) s[c] = __uint_as_float(sr[c]);
+                if (j >= mask_from) {
+                    const int lim = qp - j * kBlockN - col0;
+#pragma unroll
+                    for (int c = 0; c < 64; ++c)
+                        if (c > lim) s[c] = -INFINITY;
+                }
+                float mx4[4] = {s[0], s[1], s[2], s[3]};
+#pragma unroll
+                for (int c = 4; c < 64; c += 4) {
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) mx4[q] = fmaxf(mx4[q], s[c + q]);
+                }
+                slot[half * 128 + m] = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
             }
-            float mx = s[0];
-#pragma unroll
-            for (int c = 1; c < 128; ++c) mx = fmaxf(mx, s[c]);
+            if (named_bar_red_or(1, 256, !ok)) {
+                ok = false;
+                *abort = 1;
+                break;
+            }
+            const float mx = fmaxf(slot[m], slot[128 + m]);
             const float mx2 = mx * p.scale_log2;
             const bool grow = (m_run == -INFINITY) || (mx2 > m_run + 8.0f);
             float alpha = 1.0f;
@@ -304,35 +345,37 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
                 l_run *= alpha;
                 m_run = mx2;
             }
-            // P_j = exp2(s * scale * log2(e) - m_run), packed bf16 over columns [0, 64)
-            float psum = 0.0f;
+            // this half of P_j = exp2(s * scale * log2(e) - m_run), packed bf16 into
+            // columns [32h, 32h+32) of S_j's buffer; affine step and sum in fp32x2
+            const float2 sc2 = make_float2(p.scale_log2, p.scale_log2);
+            const float2 nm2 = make_float2(-m_run, -m_run);
+            float2 psum = make_float2(0.0f, 0.0f);
+            uint32_t pk[32];
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                uint32_t pk[16];
-#pragma unroll
-                for (int e = 0; e < 16; ++e) {
-                    const float p0 = __uint_as_float(ex2_approx(__fmaf_rn(s[c * 32 + 2 * e], p.scale_log2, -m_run)));
-                    const float p1 = __uint_as_float(ex2_approx(__fmaf_rn(s[c * 32 + 2 * e + 1], p.scale_log2, -m_run)));
-                    psum += p0 + p1;
-                    pk[e] = pack_bf16x2(p0, p1);
-                }
-                tmem_st16(lane_base + b * 128 + c * 16, pk);
+            for (int e = 0; e < 32; ++e) {
+                const float2 tt = __ffma2_rn(make_float2(s[2 * e], s[2 * e + 1]), sc2, nm2);
+                const float2 pe = make_float2(__uint_as_float(ex2_approx(tt.x)),
+                                              __uint_as_float(ex2_approx(tt.y)));
+                psum = __fadd2_rn(psum, pe);
+                pk[e] = pack_bf16x2(pe.x, pe.y);
             }
-            l_run += psum;
-            // rescale O when any row of this warp raised its max (O holds PV_0..PV_{j-1})
+            tmem_st32(lane_base + b * kBlockN + 32 * half, pk);
+            l_run += psum.x + psum.y;
+            // rescale this half of O when any row of the warp raised its max
+            // (O holds PV_0 .. PV_{j-1})
             if (j > 0 && __any_sync(0xFFFFFFFFu, grow)) {
-                const bool o_ok = mbar_wait_bounded(&bars->o_done, (j - 1) & 1, abort, p.status,
+                const bool o_ok = mbar_wait_bounded(&bars->pv_done[(j - 1) % kSBufs],
+                                                    ((j - 1) / kSBufs) & 1, abort, p.status,
                                                     kSiteAttnSoftmax, kWaitLimitNs);
-                if (!__all_sync(0xFFFFFFFFu, o_ok)) { ok = false; *abort = 1; break; }
-                tc_fence_after();
+                ok = __all_sync(0xFFFFFFFFu, o_ok);
+                if (ok) {
+                    tc_fence_after();
+                    uint32_t orr[64];
+                    tmem_ld64(lane_base + kColO + col0, orr);
 #pragma unroll
-                for (int c = 0; c < 4; ++c) {
-                    uint32_t rr[32];
-                    tmem_ld32(lane_base + kColO + c * 32, rr);
-#pragma unroll
-                    for (int e = 0; e < 32; ++e)
-                        rr[e] = __float_as_uint(__uint_as_float(rr[e]) * alpha);
-                    tmem_st32(lane_base + kColO + c * 32, rr);
+                    for (int e = 0; e < 64; ++e)
+                        orr[e] = __float_as_uint(__uint_as_float(orr[e]) * alpha);
+                    tmem_st64(lane_base + kColO + col0, orr);
                 }
             }
             tc_fence_before();
@@ -343,29 +386,34 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
                                                 kSiteAttnSoftmax, kWaitLimitNs);
             ok = __all_sync(0xFFFFFFFFu, w_ok);
         }
-        if (ok) {
+        // combine the two halves' row sums (slot 0 of the exchange array; every
+        // thread has passed its last read of it)
+        named_bar_sync(1, 256);
+        xchg[half * 128 + m] = l_run;
+        const bool fail = named_bar_red_or(1, 256, !ok || *abort);
+        const float l_tot = xchg[m] + xchg[128 + m];
+        if (!fail) {
             tc_fence_after();
-            const float inv = 1.0f / l_run;
-            __nv_bfloat16 *orow = p.o + ((static_cast<long long>(l) * p.M + r) * p.hq + g * p.G + hh) * 128;
+            const float inv = 1.0f / l_tot;
+            uint32_t orr[64];
+            tmem_ld64(lane_base + kColO + col0, orr);
+            if (valid) {
+                __nv_bfloat16 *orow =
+                    p.o + ((static_cast<long long>(l) * p.M + r) * p.hq + g * p.G + hh) * 128 + col0;
+                uint4 *dst = reinterpret_cast<uint4 *>(orow);
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                uint32_t rr[32];
-                tmem_ld32(lane_base + kColO + c * 32, rr);
-                if (valid) {
-                    uint32_t pk[16];
+                for (int e = 0; e < 8; ++e) {
+                    uint32_t w4[4];
 #pragma unroll
-                    for (int e = 0; e < 16; ++e)
-                        pk[e] = pack_bf16x2(__uint_as_float(rr[2 * e]) * inv,
-                                            __uint_as_float(rr[2 * e + 1]) * inv);
-                    uint4 *dst = reinterpret_cast<uint4 *>(orow + c * 32);
-#pragma unroll
-                    for (int e = 0; e < 4; ++e)
-                        dst[e] = make_uint4(pk[4 * e], pk[4 * e + 1], pk[4 * e + 2], pk[4 * e + 3]);
+                    for (int q = 0; q < 4; ++q)
+                        w4[q] = pack_bf16x2(__uint_as_float(orr[8 * e + 2 * q]) * inv,
+                                            __uint_as_float(orr[8 * e + 2 * q + 1]) * inv);
+                    dst[e] = make_uint4(w4[0], w4[1], w4[2], w4[3]);
                 }
+                if (half == 0 && p.lse != nullptr)
+                    p.lse[(static_cast<long long>(l) * p.M + r) * p.hq + g * p.G + hh] =
+                        (m_run + __log2f(l_tot)) * 0.69314718055994531f;
             }
-            if (valid && p.lse != nullptr)
-                p.lse[(static_cast<long long>(l) * p.M + r) * p.hq + g * p.G + hh] =
-                    (m_run + __log2f(l_run)) * 0.69314718055994531f;
         }
     }
     // tensor memory is released only after every tensor-core operation retired
@@ -428,7 +476,7 @@ cs_status launch_attn_tc(const AttnArgs &a, cudaStream_t s) {
     const cuuint64_t kdims[4] = {128, static_cast<cuuint64_t>(a.hkv), static_cast<cuuint64_t>(a.T),
                                  static_cast<cuuint64_t>(a.n_layers)};
     const cuuint64_t kstr[3] = {256ull, 256ull * a.hkv, 2ull * static_cast<cuuint64_t>(a.kv_layer_stride)};
-    const cuuint32_t kbox[4] = {64, 1, 128, 1};
+    const cuuint32_t kbox[4] = {64, 1, static_cast<cuuint32_t>(kBlockN), 1};
     if (!make_map(enc, &tq, a.q, qdims, qstr, qbox) || !make_map(enc, &tk, a.k, kdims, kstr, kbox) ||
         !make_map(enc, &tv, a.v, kdims, kstr, kbox))
         return fail(CS_ERR_INVALID_ARG, "tensor map encoding failed (alignment or extent)");

@@ -7,8 +7,8 @@
 // theta_i / (2 pi) as a 64-bit fixed-point fraction of a turn, so
 // Delta * step_i (mod 2^64) is the angle reduced to one turn, exactly up to
 // the 2^-64 rounding of step_i.  cos and sin of that angle are evaluated in
-// double-float arithmetic (~2^-45 relative), once per distinct
-// (Delta, pair) of a CTA's tokens, and kept in shared memory.
+// double-float arithmetic (~2^-45 relative), once per CTA for each distinct
+// token delta, and kept in shared memory.
 //
 // Rounding.  A bf16 output is the exact rotation rounded once to bfloat16.
 // The fast path evaluates x*c - y*s in fp32 with a proven error bound and
@@ -16,6 +16,8 @@
 // the fp32 result (Ziv's rounding test); otherwise it re-evaluates in
 // double-float and rounds that.  fp32 outputs always use the double-float
 // result.
+#include <algorithm>
+
 #include "cs_device.cuh"
 #include "cs_internal.h"
 
@@ -23,7 +25,8 @@ namespace cs {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kMaxTokensPerCta = 32;
+constexpr int kMaxTokensPerCta = 32;   // fp32 kernel
+constexpr int kMaxTokensBf16 = 8;      // bf16 kernel: token block of 8 / n_kv_heads
 
 // 1/n! split exactly into fp32 hi + lo (hi = fp32(1/n!), lo = fp32(1/n! - hi)).
 __device__ __forceinline__ f2 cf(float hi, float lo) { return {hi, lo}; }
@@ -73,21 +76,10 @@ __device__ void sincos_turns(unsigned long long u, f2 &sn, f2 &cs) {
     }
 }
 
-// bf16 bits of u*c - w*s, rounded once from the exact value.
-__device__ __forceinline__ uint32_t rot_bf16(float u, float w, float ch, float sh,
-                                             const float4 *full) {
-    const float r = __fmaf_rn(u, ch, -__fmul_rn(w, sh));
-    // |error of r| <= (|u| + |w|) * 2.5 * 2^-24 (product and fma roundings, plus
-    // |c - ch|, |s - sh| <= 2^-25); 2^-22 leaves margin for rounding E itself.
-    const float E = __fmul_rn(__fadd_rn(fabsf(u), fabsf(w)), 0x1p-22f);
-    const uint32_t b = __float_as_uint(r) & 0x7FFFFFFFu;
-    const uint32_t tb = b & 0x7FFF0000u;
-    const float mid = __uint_as_float(tb | 0x8000u);
-    const float dist = fabsf(__fsub_rn(__uint_as_float(b), mid));
-    if (dist > E && __fmul_rn(E, 1024.0f) < __uint_as_float(tb) && tb < 0x7F800000u)
-        return bf16_rne_bits(r);
-    // double-float re-evaluation
-    const float4 cs4 = *full;   // (c_hi, c_lo, s_hi, s_lo)
+// bf16 bits of u*c - w*s from the double-float evaluation (c = c_hi + c_lo,
+// s = s_hi + s_lo), rounded once: the error-free products and sum carry the
+// value to about 2^-44 relative, far inside any rounding decision left to it.
+__device__ __forceinline__ uint32_t rot_bf16_df(float u, float w, float4 cs4) {
     const f2 p = two_prod(u, cs4.x);
     const f2 q = two_prod(w, cs4.z);
     const f2 d = two_sum(p.hi, -q.hi);
@@ -95,6 +87,34 @@ __device__ __forceinline__ uint32_t rot_bf16(float u, float w, float ch, float s
                                  __fsub_rn(__fmul_rn(u, cs4.y), __fmul_rn(w, cs4.w)));
     const f2 rr = two_sum(d.hi, tail);
     return bf16_round_f2(rr.hi, rr.lo);
+}
+
+struct Row8 {
+    uint32_t w[8];   // 4 words of first-half outputs, then 4 of second-half outputs
+};
+
+// One thread's slice (8 pairs) rotated entirely in double-float and rounded
+// once; kept out of line because only a few slices in ten thousand need it.
+__device__ __noinline__ Row8 rot_row_df(uint4 xv, uint4 yv, const float4 *full) {
+    const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w};
+    const uint32_t yw[4] = {yv.x, yv.y, yv.z, yv.w};
+    Row8 out;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+        const float xa = bf16_lo(xw[w]), xb = bf16_hi(xw[w]);
+        const float ya = bf16_lo(yw[w]), yb = bf16_hi(yw[w]);
+        const float4 ca = full[2 * w], cb = full[2 * w + 1];
+        out.w[w] = rot_bf16_df(xa, ya, ca) | (rot_bf16_df(xb, yb, cb) << 16);
+        out.w[4 + w] = rot_bf16_df(ya, -xa, ca) | (rot_bf16_df(yb, -xb, cb) << 16);
+    }
+    return out;
+}
+
+// Two fp32 values rounded to nearest-even bf16 and packed (lo in bits 0-15).
+__device__ __forceinline__ uint32_t pack_bf16x2_rn(float lo, float hi) {
+    uint32_t r;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+    return r;
 }
 
 // fp32 result of u*c - w*s from the double-float evaluation.
@@ -108,8 +128,10 @@ __device__ __forceinline__ float rot_f32(float u, float w, float4 cs4) {
 }
 
 // Prologue shared by both storage types: per-token deltas and the cos/sin
-// table [tokens][64 pairs] in shared memory.  Returns false when no token of
-// the CTA moves (nothing to rotate).
+// table [tokens][64 pairs] in shared memory.  Tokens of one chunk share their
+// delta, so when every token of the block has the same delta the 64 entries
+// are evaluated once and copied.  Returns false when no token of the block
+// moves (nothing to rotate).
 __device__ bool build_table(const RebaseArgs &a, int t0, int TB, int (*s_delta)[3],
                             float4 *tab) {
     for (int j = threadIdx.x; j < TB * 3; j += blockDim.x) {
@@ -118,111 +140,170 @@ __device__ bool build_table(const RebaseArgs &a, int t0, int TB, int (*s_delta)[
         s_delta[tb][ax] = (t < a.T) ? a.pos_global[3 * t + ax] - a.pos_local[3 * t + ax] : 0;
     }
     __syncthreads();
-    int any = 0;
-    for (int j = threadIdx.x; j < TB * 3; j += blockDim.x) any |= (s_delta[j / 3][j % 3] != 0);
-    if (!__syncthreads_or(any)) return false;
-    // thread j: pair i = j % 64, a run of consecutive tokens; one evaluation per
-    // distinct delta along the run (tokens of one chunk share their delta).
-    const int groups = blockDim.x / 64;
-    const int i = threadIdx.x & 63, g = threadIdx.x >> 6;
-    const int per = (TB + groups - 1) / groups;
-    const int axis = a.axis[i];
-    const unsigned long long step = a.turn_step[i];
-    int prev = 0;
-    float4 val = make_float4(1.0f, 0.0f, 0.0f, 0.0f);
-    bool have = false;
-    for (int tb = g * per; tb < min(TB, (g + 1) * per); ++tb) {
-        const int d = s_delta[tb][axis];
-        if (!have || d != prev) {
-            if (d == 0) {
-                val = make_float4(1.0f, 0.0f, 0.0f, 0.0f);
-            } else {
-                f2 sn, cs;
-                sincos_turns(static_cast<unsigned long long>(static_cast<long long>(d)) * step,
-                             sn, cs);
-                val = make_float4(cs.hi, cs.lo, sn.hi, sn.lo);
-            }
-            prev = d;
-            have = true;
+    int any = 0, same = 1;
+    for (int j = threadIdx.x; j < TB * 3; j += blockDim.x) {
+        any |= (s_delta[j / 3][j % 3] != 0);
+        same &= (s_delta[j / 3][j % 3] == s_delta[0][j % 3]);
+    }
+    any = __syncthreads_or(any);
+    same = __syncthreads_and(same);
+    if (!any) return false;
+    const int ntok = same ? 1 : TB;
+    for (int j = threadIdx.x; j < ntok * 64; j += blockDim.x) {
+        const int tb = j >> 6, i = j & 63;
+        const int d = s_delta[tb][a.axis[i]];
+        float4 val = make_float4(1.0f, 0.0f, 0.0f, 0.0f);
+        if (d != 0) {
+            f2 sn, cs;
+            sincos_turns(static_cast<unsigned long long>(static_cast<long long>(d)) * a.turn_step[i],
+                         sn, cs);
+            val = make_float4(cs.hi, cs.lo, sn.hi, sn.lo);
         }
-        tab[tb * 64 + i] = val;
+        if (same) {
+            for (int q = 0; q < TB; ++q) tab[q * 64 + i] = val;
+        } else {
+            tab[tb * 64 + i] = val;
+        }
     }
     __syncthreads();
     return true;
 }
 
-// bf16: 8 threads per 128-element row, each owning 8 frequency pairs
-// (16 bytes of the first half and the matching 16 bytes of the second half).
-__global__ void __launch_bounds__(kThreads) rebase_bf16_kernel(RebaseArgs a, int layers_per_cta) {
-    __shared__ float4 tab[kMaxTokensPerCta * 64];
-    __shared__ int s_delta[kMaxTokensPerCta][3];
-    const int TB = max(1, kMaxTokensPerCta / a.hkv);
+// Rotates one thread's slice: 8 frequency pairs, i.e. 16-byte words xv (first
+// half: elements i) and yv (second half: elements i + 64).  Returns false if
+// the bf16 rounding of any output is uncertain.
+//
+// Each output r ~ u c - w s is evaluated in fp32 with |error| <= E, where
+// E = (|x| + |y|) * 2.5 * 2^-24 (product and fma roundings plus
+// |c - c_hi|, |s - s_hi| <= 2^-25), bounded here by (|x| + |y|) * 2^-22.  The
+// bf16 rounding is certain when no bf16 midpoint lies within E of r: the
+// midpoint of r's interval is (|r| truncated to bf16) + half a bf16 unit, an
+// fp32 number in r's binade, so |r| - mid is exact; requiring |r| > 2048 E
+// keeps the neighbouring intervals' midpoints (at least |r| / 1024 away) out
+// of reach too.  A NaN or infinite r fails.
+__device__ __forceinline__ bool rotate_slice(const uint4 &xv, const uint4 &yv, const float (&c)[8],
+                                             const float (&sn)[8], uint32_t (&ow)[4],
+                                             uint32_t (&pw)[4]) {
+    const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w};
+    const uint32_t yw[4] = {yv.x, yv.y, yv.z, yv.w};
+    bool ok = true;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+        float r1[2], r2[2];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const int e = 2 * w + h;
+            const float x = h ? bf16_hi(xw[w]) : bf16_lo(xw[w]);
+            const float y = h ? bf16_hi(yw[w]) : bf16_lo(yw[w]);
+            r1[h] = __fmaf_rn(x, c[e], -__fmul_rn(y, sn[e]));    // x c - y s
+            r2[h] = __fmaf_rn(y, c[e], __fmul_rn(x, sn[e]));     // y c + x s
+            const float E = __fmul_rn(__fadd_rn(fabsf(x), fabsf(y)), 0x1p-22f);
+            const float E2 = __fmul_rn(E, 2048.0f);
+            const float m1 = __uint_as_float((__float_as_uint(r1[h]) & 0x7FFF0000u) | 0x8000u);
+            const float m2 = __uint_as_float((__float_as_uint(r2[h]) & 0x7FFF0000u) | 0x8000u);
+            ok = ok & (fabsf(__fsub_rn(fabsf(r1[h]), m1)) > E) & (fabsf(r1[h]) > E2) &
+                 (fabsf(__fsub_rn(fabsf(r2[h]), m2)) > E) & (fabsf(r2[h]) > E2);
+        }
+        ow[w] = pack_bf16x2_rn(r1[0], r1[1]);
+        pw[w] = pack_bf16x2_rn(r2[0], r2[1]);
+    }
+    return ok;
+}
+
+// bf16: 8 threads per 128-element row, each owning 8 frequency pairs (16 bytes
+// of the first half and the matching 16 bytes of the second half).  A CTA
+// takes a block of TB tokens (TB * n_kv_heads * 8 threads per layer "slot")
+// and walks every layer of its range, n_slots layers at a time, so the cos/sin
+// table of its tokens is built once and reused across layers.
+//   - each thread reads its own token's delta and issues its first load before
+//     the table is built, so DRAM latency overlaps the sincos evaluation;
+//   - the next layer's slice is loaded before the current one is rotated;
+//   - a slice with an uncertain rounding is not stored; its layer is recorded
+//     and, after the streaming loop, redone in double-float from the untouched
+//     input (keeping the rare slow path out of the hot loop).
+__global__ void __launch_bounds__(kThreads, 4) rebase_bf16_kernel(RebaseArgs a, int TB, int l_per_cta) {
+    __shared__ float4 tab[kMaxTokensBf16 * 64];
+    __shared__ int s_delta[kMaxTokensBf16][3];
     const int t0 = blockIdx.x * TB;
-    const int l0 = blockIdx.y * layers_per_cta;
-    const int l1 = min(a.n_layers, l0 + layers_per_cta);
-    const bool moved_any = build_table(a, t0, TB, s_delta, tab);
-    if (!moved_any && a.in_place) return;
-
-    const int slot = threadIdx.x;
-    if (slot >= TB * a.hkv * 8) return;
-    const int tb = slot / (a.hkv * 8);
-    const int h = (slot >> 3) % a.hkv;
-    const int pg = slot & 7;
+    const int l0 = blockIdx.y * l_per_cta;
+    const int l1 = min(a.n_layers, l0 + l_per_cta);
+    const int slot_threads = TB * a.hkv * 8;
+    const int n_slots = kThreads / slot_threads;
+    const int slot = threadIdx.x / slot_threads;
+    const int loc = threadIdx.x - slot * slot_threads;
+    const int tb = loc / (a.hkv * 8);
+    const int h = (loc >> 3) % a.hkv;
+    const int pg = loc & 7;
     const int t = t0 + tb;
-    if (t >= a.T) return;
-    const bool moved = (s_delta[tb][0] | s_delta[tb][1] | s_delta[tb][2]) != 0;
-    if (!moved && a.in_place) return;
-
+    const int lfirst = l0 + slot;
+    bool mine = (slot < n_slots) && (t < a.T) && (lfirst < l1);
+    bool moved = false;
+    if (mine) {
+        moved = ((a.pos_global[3 * t] - a.pos_local[3 * t]) |
+                 (a.pos_global[3 * t + 1] - a.pos_local[3 * t + 1]) |
+                 (a.pos_global[3 * t + 2] - a.pos_local[3 * t + 2])) != 0;
+        if (!moved && a.in_place) mine = false;
+    }
+    const int count = mine ? (l1 - lfirst + n_slots - 1) / n_slots : 0;
     const __nv_bfloat16 *src = static_cast<const __nv_bfloat16 *>(a.k_in);
     __nv_bfloat16 *dst = static_cast<__nv_bfloat16 *>(a.k_out);
     const long long row0 = (static_cast<long long>(t) * a.hkv + h) * 128 + pg * 8;
+    const long long lstep = static_cast<long long>(n_slots) * a.layer_stride;
+    const long long obase = static_cast<long long>(lfirst) * a.layer_stride + row0;
+    uint4 xv = make_uint4(0, 0, 0, 0), yv = make_uint4(0, 0, 0, 0);
+    if (count > 0) {
+        xv = __ldcs(reinterpret_cast<const uint4 *>(src + obase));
+        yv = __ldcs(reinterpret_cast<const uint4 *>(src + obase + 64));
+    }
+    const bool moved_any = build_table(a, t0, TB, s_delta, tab);
+    if (count == 0) return;
+    if (!moved) {   // out-of-place copy of an unmoved token
+        for (int i = 0; i < count; ++i) {
+            const long long o = obase + i * lstep;
+            if (i > 0) {
+                xv = __ldcs(reinterpret_cast<const uint4 *>(src + o));
+                yv = __ldcs(reinterpret_cast<const uint4 *>(src + o + 64));
+            }
+            __stcs(reinterpret_cast<uint4 *>(dst + o), xv);
+            __stcs(reinterpret_cast<uint4 *>(dst + o + 64), yv);
+        }
+        return;
+    }
+    (void)moved_any;   // a moved token implies the table was built
     const float4 *full = &tab[tb * 64 + pg * 8];
-    float ch[8], sh[8];
+    float c[8], sn[8];
 #pragma unroll
     for (int e = 0; e < 8; ++e) {
-        const float4 v = full[e];
-        ch[e] = v.x;
-        sh[e] = v.z;
+        c[e] = full[e].x;
+        sn[e] = full[e].z;
     }
-    for (int l = l0; l < l1; l += 2) {
-        const bool two = (l + 1 < l1);
-        const long long o0 = static_cast<long long>(l) * a.layer_stride + row0;
-        const long long o1 = o0 + a.layer_stride;
-        uint4 x0 = __ldcs(reinterpret_cast<const uint4 *>(src + o0));
-        uint4 y0 = __ldcs(reinterpret_cast<const uint4 *>(src + o0 + 64));
-        uint4 x1 = make_uint4(0, 0, 0, 0), y1 = make_uint4(0, 0, 0, 0);
-        if (two) {
-            x1 = __ldcs(reinterpret_cast<const uint4 *>(src + o1));
-            y1 = __ldcs(reinterpret_cast<const uint4 *>(src + o1 + 64));
+    unsigned long long redo = 0;   // the host keeps count <= 64
+    for (int i = 0; i < count; ++i) {
+        uint4 xn = make_uint4(0, 0, 0, 0), yn = make_uint4(0, 0, 0, 0);
+        if (i + 1 < count) {
+            xn = __ldcs(reinterpret_cast<const uint4 *>(src + obase + (i + 1) * lstep));
+            yn = __ldcs(reinterpret_cast<const uint4 *>(src + obase + (i + 1) * lstep + 64));
         }
-        for (int rep = 0; rep < (two ? 2 : 1); ++rep) {
-            const uint4 xv = rep ? x1 : x0, yv = rep ? y1 : y0;
-            const long long o = rep ? o1 : o0;
-            if (!moved) {   // out-of-place copy of an unmoved token
-                __stcs(reinterpret_cast<uint4 *>(dst + o), xv);
-                __stcs(reinterpret_cast<uint4 *>(dst + o + 64), yv);
-                continue;
-            }
-            const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w};
-            const uint32_t yw[4] = {yv.x, yv.y, yv.z, yv.w};
-            uint32_t ow[4], pw[4];
-#pragma unroll
-            for (int w = 0; w < 4; ++w) {
-                const int e0 = 2 * w, e1 = 2 * w + 1;
-                const float xa = bf16_lo(xw[w]), xb = bf16_hi(xw[w]);
-                const float ya = bf16_lo(yw[w]), yb = bf16_hi(yw[w]);
-                // first half: x c - y s ; second half: y c + x s = y c - (-x) s
-                const uint32_t r0 = rot_bf16(xa, ya, ch[e0], sh[e0], full + e0);
-                const uint32_t r1 = rot_bf16(xb, yb, ch[e1], sh[e1], full + e1);
-                const uint32_t q0 = rot_bf16(ya, -xa, ch[e0], sh[e0], full + e0);
-                const uint32_t q1 = rot_bf16(yb, -xb, ch[e1], sh[e1], full + e1);
-                ow[w] = r0 | (r1 << 16);
-                pw[w] = q0 | (q1 << 16);
-            }
+        uint32_t ow[4], pw[4];
+        if (rotate_slice(xv, yv, c, sn, ow, pw)) {
+            const long long o = obase + i * lstep;
             __stcs(reinterpret_cast<uint4 *>(dst + o), make_uint4(ow[0], ow[1], ow[2], ow[3]));
-            __stcs(reinterpret_cast<uint4 *>(dst + o + 64),
-                   make_uint4(pw[0], pw[1], pw[2], pw[3]));
+            __stcs(reinterpret_cast<uint4 *>(dst + o + 64), make_uint4(pw[0], pw[1], pw[2], pw[3]));
+        } else {
+            redo |= 1ull << i;
         }
+        xv = xn;
+        yv = yn;
+    }
+    while (redo) {   // rare: slices whose rounding was uncertain, redone in double-float
+        const int i = __ffsll(static_cast<long long>(redo)) - 1;
+        redo &= redo - 1;
+        const long long o = obase + i * lstep;
+        const uint4 x0 = *reinterpret_cast<const uint4 *>(src + o);
+        const uint4 y0 = *reinterpret_cast<const uint4 *>(src + o + 64);
+        const Row8 rr = rot_row_df(x0, y0, full);
+        *reinterpret_cast<uint4 *>(dst + o) = make_uint4(rr.w[0], rr.w[1], rr.w[2], rr.w[3]);
+        *reinterpret_cast<uint4 *>(dst + o + 64) = make_uint4(rr.w[4], rr.w[5], rr.w[6], rr.w[7]);
     }
 }
 
@@ -277,15 +358,28 @@ __global__ void __launch_bounds__(kThreads) rebase_f32_kernel(RebaseArgs a, int 
 
 cudaError_t launch_rebase(const RebaseArgs &a, cs_dtype dt, cudaStream_t s) {
     if (a.T == 0 || a.n_layers == 0) return cudaSuccess;
-    const bool bf = (dt == CS_DTYPE_BF16);
-    const int TB = bf ? (a.hkv >= kMaxTokensPerCta ? 1 : kMaxTokensPerCta / a.hkv)
-                      : (a.hkv >= kMaxTokensPerCta / 2 ? 1 : (kMaxTokensPerCta / 2) / a.hkv);
-    const int layers_per_cta = 4;
-    dim3 grid((a.T + TB - 1) / TB, (a.n_layers + layers_per_cta - 1) / layers_per_cta);
-    if (bf)
-        rebase_bf16_kernel<<<grid, kThreads, 0, s>>>(a, layers_per_cta);
-    else
+    if (dt == CS_DTYPE_BF16) {
+        // token block: 64 threads per layer slot where possible (4 slots per CTA)
+        const int TB = a.hkv >= 8 ? 1 : 8 / a.hkv;
+        const int blocks = (a.T + TB - 1) / TB;
+        const int slots = kThreads / (TB * a.hkv * 8);
+        // split layers across CTAs only when there are too few token blocks to fill
+        // the GPU (every extra CTA repeats the cos/sin prologue)
+        int groups = 1;
+        const int target = 152 * 2;
+        if (blocks < target) groups = std::min((target + blocks - 1) / blocks,
+                                               (a.n_layers + slots - 1) / slots);
+        // each thread walks at most 64 layers (its redo mask is 64 bits)
+        groups = std::max(groups, (a.n_layers + 64 * slots - 1) / (64 * slots));
+        const int l_per_cta = (a.n_layers + groups - 1) / groups;
+        dim3 grid(blocks, (a.n_layers + l_per_cta - 1) / l_per_cta);
+        rebase_bf16_kernel<<<grid, kThreads, 0, s>>>(a, TB, l_per_cta);
+    } else {
+        const int TB = a.hkv >= kMaxTokensPerCta / 2 ? 1 : (kMaxTokensPerCta / 2) / a.hkv;
+        const int layers_per_cta = 4;
+        dim3 grid((a.T + TB - 1) / TB, (a.n_layers + layers_per_cta - 1) / layers_per_cta);
         rebase_f32_kernel<<<grid, kThreads, 0, s>>>(a, layers_per_cta);
+    }
     return cudaGetLastError();
 }
 

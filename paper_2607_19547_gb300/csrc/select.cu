@@ -15,13 +15,14 @@ namespace {
 constexpr int kThreads = 1024;
 constexpr int kWarps = kThreads / 32;
 
-__device__ __forceinline__ uint32_t order_key(float f) {
-    const uint32_t u = __float_as_uint(f);
+// Order-preserving key of an fp32 bit pattern u (scores are read as raw 32-bit
+// words, never as floats, so every NaN payload and sign survives).
+__device__ __forceinline__ uint32_t order_key(uint32_t u) {
     return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
-select_kernel(const float *__restrict__ score, int n, int k, int idx_base, int *__restrict__ out) {
+select_kernel(const uint32_t *__restrict__ score, int n, int k, int idx_base, int *__restrict__ out) {
     __shared__ uint32_t hist[kWarps][256];
     __shared__ uint32_t total[256];
     __shared__ uint32_t s_digit, s_krem;
@@ -119,7 +120,8 @@ select_kernel(const float *__restrict__ score, int n, int k, int idx_base, int *
 cudaError_t launch_select(const float *score, int n, int k, int idx_base, int *out,
                           cudaStream_t s) {
     if (k == 0 || n == 0) return cudaSuccess;
-    select_kernel<<<1, kThreads, 0, s>>>(score, n, k, idx_base, out);
+    select_kernel<<<1, kThreads, 0, s>>>(reinterpret_cast<const uint32_t *>(score), n, k, idx_base,
+                                         out);
     return cudaGetLastError();
 }
 
