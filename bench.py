@@ -45,6 +45,20 @@ def _dist_env():
     return ws, rank, local
 
 
+def max_over_ranks(x: float, device) -> float:
+    """The largest value of x over all ranks (x itself with a single process)."""
+    if not (torch.distributed.is_available() and torch.distributed.is_initialized()):
+        return float(x)
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def replica_throughput(units_per_replica: float, ms_slowest: float, world: int) -> float:
+    """Whole-job throughput of `world` independent replicas timed by the slowest one."""
+    return world * units_per_replica / (ms_slowest / 1e3)
+
+
 def peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(path):
@@ -183,12 +197,8 @@ def run_gpu(args, w, ws, rank, local):
     per = np.array([[events[i][j].elapsed_time(events[i][j + 1]) for j in range(4)]
                     for i in range(args.steps)])   # ms: rebase, score, select, attention
     step_ms = per.sum(axis=1)
-    ms_per_step = float(step_ms.mean())
-    if ws > 1:
-        t = torch.tensor([ms_per_step], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms_per_step = float(t.item())
-    value = ws * w.t_vis / (ms_per_step / 1e3)
+    ms_per_step = max_over_ranks(float(step_ms.mean()), dev)
+    value = replica_throughput(w.t_vis, ms_per_step, ws)
 
     qpos = q.qpos.cpu().numpy()
     pk = peaks()
@@ -240,11 +250,7 @@ def run_gpu(args, w, ws, rank, local):
         torch.cuda.synchronize()
         e2e_ms.append(e0.elapsed_time(e1))
     cs.cs_sync_status()
-    e2e_mean = float(np.mean(e2e_ms))
-    if ws > 1:
-        t = torch.tensor([e2e_mean], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        e2e_mean = float(t.item())
+    e2e_mean = max_over_ranks(float(np.mean(e2e_ms)), dev)
     line = {
         "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": ws,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 5),
@@ -260,7 +266,7 @@ def run_gpu(args, w, ws, rank, local):
                    "parallelism": f"{ws} independent replica(s)"},
         "roofline": roofline,
         "kernels": kernels,
-        "e2e": {"value": round(ws * w.t_vis / (e2e_mean / 1e3), 1), "unit": UNIT,
+        "e2e": {"value": round(replica_throughput(w.t_vis, e2e_mean, ws), 1), "unit": UNIT,
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "ms_per_step": round(e2e_mean, 4)},
         "gpu_launches": 4 * args.steps,
