@@ -28,7 +28,8 @@
 //               updates the running max (rescaling its half of O in TMEM only
 //               when the max grows by more than 2^8), writes its half of
 //               P_j = exp2(...) as bf16 over S_j's TMEM columns, and finally
-//               normalises its half of O and stores it.
+//               normalises its half of O into the Q tile's shared memory (idle
+//               after the last S), from where two TMA stores write whole rows.
 // TMEM: S buffers at columns 0, 128, 256; O at 384.  S_j reuses the buffer
 // of P_{j-3}, so the S issuer runs up to three blocks ahead of the softmax.
 // Every mbarrier wait is bounded; on a timeout the CTA records
@@ -126,7 +127,8 @@ __device__ __forceinline__ int clamp_pos(int x, int T) { return min(max(x, 0), T
 
 __global__ void __launch_bounds__(kThreads, 1)
 attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
-               const __grid_constant__ CUtensorMap tm_v, const TcParams p) {
+               const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_o,
+               const TcParams p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *base = reinterpret_cast<uint8_t *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -162,6 +164,16 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
         mbar_init(&bars->mma_done, 2);
         bars->abort = 0;
         fence_mbar_init();
+        // thread 0 is the Q/K producer: Q and the first K block go out before the
+        // CTA-wide barrier (nothing else touches these barriers until after it)
+        tma_prefetch_desc(&tm_q);
+        tma_prefetch_desc(&tm_k);
+        mbar_arrive_expect_tx(&bars->q_full, q_bytes);
+        tma_load_4d(base + Smem::q, &tm_q, &bars->q_full, 0, g * p.G, r0, l);
+        tma_load_4d(base + Smem::q + kHalf, &tm_q, &bars->q_full, 64, g * p.G, r0, l);
+        mbar_arrive_expect_tx(&bars->k_full[0], kTileBytes);
+        tma_load_4d(base + Smem::k, &tm_k, &bars->k_full[0], 0, g, 0, l);
+        tma_load_4d(base + Smem::k + kHalf, &tm_k, &bars->k_full[0], 64, g, 0, l);
     }
     if (warp == 1) {
         tmem_alloc(&bars->tmem_base, kTmemCols);
@@ -184,23 +196,17 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
 
     if (warp == 0) {
         // ------------------------------------------------------------ producers
-        // lane 0 streams Q and the K ring, lane 1 the V ring
+        // lane 0 streams the K ring (Q and K block 0 went out at set-up), lane 1 the V ring
         if (lane < 2) {
             volatile int never = 0;
-            int issued = 0;
+            int issued = lane == 0 ? 1 : 0;
             const int stages = lane == 0 ? kKStages : kVStages;
             uint64_t *full = lane == 0 ? bars->k_full : bars->v_full;
             uint64_t *empty = lane == 0 ? bars->k_empty : bars->v_empty;
             const CUtensorMap *tm = lane == 0 ? &tm_k : &tm_v;
             const uint32_t ring = lane == 0 ? Smem::k : Smem::v;
-            tma_prefetch_desc(tm);
-            if (lane == 0) {
-                tma_prefetch_desc(&tm_q);
-                mbar_arrive_expect_tx(&bars->q_full, q_bytes);
-                tma_load_4d(base + Smem::q, &tm_q, &bars->q_full, 0, g * p.G, r0, l);
-                tma_load_4d(base + Smem::q + kHalf, &tm_q, &bars->q_full, 64, g * p.G, r0, l);
-            }
-            for (int j = 0; j < nb; ++j) {
+            if (lane == 1) tma_prefetch_desc(tm);
+            for (int j = issued; j < nb; ++j) {
                 const int s = j % stages;
                 if (!mbar_wait_bounded(&empty[s], ((j / stages) & 1) ^ 1, abort, p.status,
                                        kSiteAttnProducer, kWaitLimitNs)) break;
@@ -397,23 +403,31 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
             const float inv = 1.0f / l_tot;
             uint32_t orr[64];
             tmem_ld64(lane_base + kColO + col0, orr);
-            if (valid) {
-                __nv_bfloat16 *orow =
-                    p.o + ((static_cast<long long>(l) * p.M + r) * p.hq + g * p.G + hh) * 128 + col0;
-                uint4 *dst = reinterpret_cast<uint4 *>(orow);
+            // O leaves through shared memory: the Q tile (no MMA reads it after the last
+            // S) in the same 128-byte-swizzled layout, then one TMA store per half, so
+            // the global writes are whole rows; rows past M are clipped by the store
+            uint8_t *orow = base + Smem::q + half * kHalf + m * 128;
 #pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    uint32_t w4[4];
+            for (int e = 0; e < 8; ++e) {
+                uint32_t w4[4];
 #pragma unroll
-                    for (int q = 0; q < 4; ++q)
-                        w4[q] = pack_bf16x2(__uint_as_float(orr[8 * e + 2 * q]) * inv,
-                                            __uint_as_float(orr[8 * e + 2 * q + 1]) * inv);
-                    dst[e] = make_uint4(w4[0], w4[1], w4[2], w4[3]);
-                }
-                if (half == 0 && p.lse != nullptr)
-                    p.lse[(static_cast<long long>(l) * p.M + r) * p.hq + g * p.G + hh] =
-                        (m_run + __log2f(l_tot)) * 0.69314718055994531f;
+                for (int q = 0; q < 4; ++q)
+                    w4[q] = pack_bf16x2(__uint_as_float(orr[8 * e + 2 * q]) * inv,
+                                        __uint_as_float(orr[8 * e + 2 * q + 1]) * inv);
+                *reinterpret_cast<uint4 *>(orow + ((e ^ (m & 7)) << 4)) =
+                    make_uint4(w4[0], w4[1], w4[2], w4[3]);
             }
+            if (valid && half == 0 && p.lse != nullptr)
+                p.lse[(static_cast<long long>(l) * p.M + r) * p.hq + g * p.G + hh] =
+                    (m_run + __log2f(l_tot)) * 0.69314718055994531f;
+            fence_proxy_async_smem();
+        }
+        named_bar_sync(1, 256);   // `fail` is the same in every softmax thread
+        if (!fail && threadIdx.x == 64) {
+            tma_store_4d(&tm_o, base + Smem::q, 0, g * p.G, r0, l);
+            tma_store_4d(&tm_o, base + Smem::q + kHalf, 64, g * p.G, r0, l);
+            bulk_commit();
+            bulk_wait_all();   // the stores have read shared memory before the CTA exits
         }
     }
     // tensor memory is released only after every tensor-core operation retired
@@ -468,7 +482,7 @@ cs_status launch_attn_tc(const AttnArgs &a, cudaStream_t s) {
     if (items > 0x7FFFFFFFll) return fail(CS_ERR_UNSUPPORTED, "too many attention tiles");
     EncodeTiledFn enc = get_encode_fn();
     if (enc == nullptr) return fail(CS_ERR_CUDA, "cuTensorMapEncodeTiled is not available");
-    CUtensorMap tq, tk, tv;
+    CUtensorMap tq, tk, tv, to;
     const cuuint64_t qdims[4] = {128, static_cast<cuuint64_t>(a.hq), static_cast<cuuint64_t>(a.M),
                                  static_cast<cuuint64_t>(a.n_layers)};
     const cuuint64_t qstr[3] = {256ull, 256ull * a.hq, 256ull * a.hq * a.M};
@@ -477,7 +491,8 @@ cs_status launch_attn_tc(const AttnArgs &a, cudaStream_t s) {
                                  static_cast<cuuint64_t>(a.n_layers)};
     const cuuint64_t kstr[3] = {256ull, 256ull * a.hkv, 2ull * static_cast<cuuint64_t>(a.kv_layer_stride)};
     const cuuint32_t kbox[4] = {64, 1, static_cast<cuuint32_t>(kBlockN), 1};
-    if (!make_map(enc, &tq, a.q, qdims, qstr, qbox) || !make_map(enc, &tk, a.k, kdims, kstr, kbox) ||
+    if (!make_map(enc, &tq, a.q, qdims, qstr, qbox) || !make_map(enc, &to, a.o, qdims, qstr, qbox) ||
+        !make_map(enc, &tk, a.k, kdims, kstr, kbox) ||
         !make_map(enc, &tv, a.v, kdims, kstr, kbox))
         return fail(CS_ERR_INVALID_ARG, "tensor map encoding failed (alignment or extent)");
     TcParams p;
@@ -502,7 +517,7 @@ cs_status launch_attn_tc(const AttnArgs &a, cudaStream_t s) {
                                         static_cast<int>(smem));
     });
     if (attr_err != cudaSuccess) return cuda_fail(attr_err, "cudaFuncSetAttribute");
-    attn_tc_kernel<<<static_cast<unsigned>(items), kThreads, smem, s>>>(tq, tk, tv, p);
+    attn_tc_kernel<<<static_cast<unsigned>(items), kThreads, smem, s>>>(tq, tk, tv, to, p);
     const cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_fail(e, "attention launch");
     return CS_OK;
