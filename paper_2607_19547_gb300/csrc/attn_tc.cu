@@ -145,35 +145,38 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
     const int mask_from = qmin / kBlockN;
     const uint32_t q_bytes = static_cast<uint32_t>(p.tok * p.G) * 256u;   // both 64-column halves
 
-    if (threadIdx.x == 0) {
-        mbar_init(&bars->q_full, 1);
-        for (int s = 0; s < kKStages; ++s) {
-            mbar_init(&bars->k_full[s], 1);
-            mbar_init(&bars->k_empty[s], 1);
+    if (warp == 0) {
+        // thread 0 is the Q/K producer: Q and the first K block go out before the other
+        // barriers are initialised and before the CTA-wide barrier (nothing else
+        // touches these barriers until after it); lanes initialise the rest in parallel
+        if (lane == 0) {
+            mbar_init(&bars->q_full, 1);
+            mbar_init(&bars->k_full[0], 1);
+            fence_mbar_init();
+            tma_prefetch_desc(&tm_q);
+            tma_prefetch_desc(&tm_k);
+            mbar_arrive_expect_tx(&bars->q_full, q_bytes);
+            tma_load_4d(base + Smem::q, &tm_q, &bars->q_full, 0, g * p.G, r0, l);
+            tma_load_4d(base + Smem::q + kHalf, &tm_q, &bars->q_full, 64, g * p.G, r0, l);
+            mbar_arrive_expect_tx(&bars->k_full[0], kTileBytes);
+            tma_load_4d(base + Smem::k, &tm_k, &bars->k_full[0], 0, g, 0, l);
+            tma_load_4d(base + Smem::k + kHalf, &tm_k, &bars->k_full[0], 64, g, 0, l);
         }
-        for (int s = 0; s < kVStages; ++s) {
-            mbar_init(&bars->v_full[s], 1);
-            mbar_init(&bars->v_empty[s], 1);
+        if (lane >= 1 && lane < kKStages) mbar_init(&bars->k_full[lane], 1);
+        if (lane < kKStages) mbar_init(&bars->k_empty[lane], 1);
+        if (lane < kVStages) {
+            mbar_init(&bars->v_full[lane], 1);
+            mbar_init(&bars->v_empty[lane], 1);
         }
-        for (int b = 0; b < kSBufs; ++b) {
-            mbar_init(&bars->s_full[b], 1);
-            mbar_init(&bars->p_full[b], 256);
-            mbar_init(&bars->pv_done[b], 1);
+        if (lane < kSBufs) {
+            mbar_init(&bars->s_full[lane], 1);
+            mbar_init(&bars->p_full[lane], 256);
+            mbar_init(&bars->pv_done[lane], 1);
         }
-        mbar_init(&bars->o_final, 1);
-        mbar_init(&bars->mma_done, 2);
-        bars->abort = 0;
+        if (lane == 8) mbar_init(&bars->o_final, 1);
+        if (lane == 9) mbar_init(&bars->mma_done, 2);
+        if (lane == 10) bars->abort = 0;
         fence_mbar_init();
-        // thread 0 is the Q/K producer: Q and the first K block go out before the
-        // CTA-wide barrier (nothing else touches these barriers until after it)
-        tma_prefetch_desc(&tm_q);
-        tma_prefetch_desc(&tm_k);
-        mbar_arrive_expect_tx(&bars->q_full, q_bytes);
-        tma_load_4d(base + Smem::q, &tm_q, &bars->q_full, 0, g * p.G, r0, l);
-        tma_load_4d(base + Smem::q + kHalf, &tm_q, &bars->q_full, 64, g * p.G, r0, l);
-        mbar_arrive_expect_tx(&bars->k_full[0], kTileBytes);
-        tma_load_4d(base + Smem::k, &tm_k, &bars->k_full[0], 0, g, 0, l);
-        tma_load_4d(base + Smem::k + kHalf, &tm_k, &bars->k_full[0], 64, g, 0, l);
     }
     if (warp == 1) {
         tmem_alloc(&bars->tmem_base, kTmemCols);
@@ -427,7 +430,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
             tma_store_4d(&tm_o, base + Smem::q, 0, g * p.G, r0, l);
             tma_store_4d(&tm_o, base + Smem::q + kHalf, 64, g * p.G, r0, l);
             bulk_commit();
-            bulk_wait_all();   // the stores have read shared memory before the CTA exits
+            bulk_wait_read();   // the stores have read shared memory before the CTA exits
         }
     }
     // tensor memory is released only after every tensor-core operation retired

@@ -196,7 +196,7 @@ __device__ __forceinline__ void tma_load_4d(void *dst, const void *desc, uint64_
 }
 
 // 4-D tiled store shared -> global (bulk async group); rows outside the tensor
-// are clipped.  Completion: bulk_commit() then bulk_wait_all().
+// are clipped.  Completion: bulk_commit() then bulk_wait_read().
 __device__ __forceinline__ void tma_store_4d(const void *desc, const void *src, int c0, int c1, int c2,
                                              int c3) {
     asm volatile(
@@ -210,8 +210,10 @@ __device__ __forceinline__ void bulk_commit() {
     asm volatile("cp.async.bulk.commit_group;" ::: "memory");
 }
 
-__device__ __forceinline__ void bulk_wait_all() {
-    asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+// Waits until every committed bulk store has finished reading shared memory
+// (the global writes complete on their own; the shared memory may be reused).
+__device__ __forceinline__ void bulk_wait_read() {
+    asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
 }
 
 // ---------------------------------------------------------------------------
