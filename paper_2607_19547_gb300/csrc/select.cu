@@ -1,11 +1,15 @@
 // Step 3 of the composition path: top-rho selection (ChronoStitch Sec. 2).
 //
-// One CTA of 1024 threads (the candidate scores are a few hundred KB and stay
-// in L2).  Scores map to order-preserving 32-bit keys; four MSB-first radix
-// passes over 8-bit digits find K*, the k-th largest key, and how many keys
-// equal to K* belong to the top k (the lowest-index ones: the tie-break).  A
-// final pass in index order writes the selected indices with a block-wide
-// prefix count, so the output is ascending without a sort.
+// One CTA of 1024 threads (the candidate scores are a few hundred KB at most and
+// stay in L2).  Scores map to order-preserving 32-bit keys.  Thread t owns the
+// contiguous candidate range [t*per, (t+1)*per); up to 16 keys per thread stay
+// in registers, larger inputs are re-read from L2 in every pass.  Three
+// MSB-first radix passes over 11-, 11- and 10-bit digits (one shared 2048-bin
+// histogram, warp-aggregated increments) find K*, the k-th largest key, and how
+// many keys equal to K* belong to the top k (the lowest-index ones: the
+// tie-break).  One block-wide scan of the per-thread (greater, equal) counts
+// then gives every selected index its output position, so the output is
+// ascending without a sort.
 #include "cs_device.cuh"
 #include "cs_internal.h"
 
@@ -14,6 +18,8 @@ namespace {
 
 constexpr int kThreads = 1024;
 constexpr int kWarps = kThreads / 32;
+constexpr int kBins = 2048;
+constexpr int kRegKeys = 16;   // keys per thread held in registers (n <= 16384)
 
 // Order-preserving key of an fp32 bit pattern u (scores are read as raw 32-bit
 // words, never as floats, so every NaN payload and sign survives).
@@ -21,97 +27,142 @@ __device__ __forceinline__ uint32_t order_key(uint32_t u) {
     return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
+// hist[d] += 1 for every lane with `active`; lanes sharing a digit add once.
+__device__ __forceinline__ void hist_add(uint32_t *hist, uint32_t d, bool active) {
+    const uint32_t am = __ballot_sync(0xFFFFFFFFu, active);
+    if (active) {
+        const uint32_t peers = __match_any_sync(am, d);
+        if ((threadIdx.x & 31) == __ffs(peers) - 1) atomicAdd(&hist[d], __popc(peers));
+    }
+}
+
+// Block-wide inclusive scan of v (all 1024 threads call; wsum holds 32 words).
+// Callers separate two uses of wsum with a barrier.
+template <typename T>
+__device__ __forceinline__ T block_incl_scan(T v, T *wsum) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+    for (int o = 1; o < 32; o *= 2) {
+        const T y = __shfl_up_sync(0xFFFFFFFFu, v, o);
+        if (lane >= o) v += y;
+    }
+    if (lane == 31) wsum[warp] = v;
+    __syncthreads();
+    if (warp == 0) {
+        T w = wsum[lane];
+#pragma unroll
+        for (int o = 1; o < 32; o *= 2) {
+            const T y = __shfl_up_sync(0xFFFFFFFFu, w, o);
+            if (lane >= o) w += y;
+        }
+        wsum[lane] = w;
+    }
+    __syncthreads();
+    return warp > 0 ? v + wsum[warp - 1] : v;
+}
+
+// KPT > 0: exactly KPT keys per thread in registers; KPT == 0: per keys per
+// thread read from global memory in every pass.
+template <int KPT>
 __global__ void __launch_bounds__(kThreads, 1)
-select_kernel(const uint32_t *__restrict__ score, int n, int k, int idx_base, int *__restrict__ out) {
-    __shared__ uint32_t hist[kWarps][256];
-    __shared__ uint32_t total[256];
+select_kernel(const uint32_t *__restrict__ score, int n, int k, int idx_base, int per,
+              int *__restrict__ out) {
+    __shared__ uint32_t hist[kBins];
+    __shared__ unsigned long long wsum[kWarps];
     __shared__ uint32_t s_digit, s_krem;
-    __shared__ uint32_t wcnt[kWarps][2];
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int tid = threadIdx.x;
 
     if (k >= n) {   // everything is selected, in index order
         for (int i = tid; i < n; i += kThreads) out[i] = idx_base + i;
         return;
     }
+    const int i0 = tid * per;
+    const int cnt = max(0, min(per, n - i0));
+    uint32_t reg[KPT > 0 ? KPT : 1];
+    if (KPT > 0) {
+#pragma unroll
+        for (int i = 0; i < (KPT > 0 ? KPT : 1); ++i)
+            reg[i] = i < cnt ? order_key(__ldg(score + i0 + i)) : 0u;
+    }
+    auto key_at = [&](int i) -> uint32_t {
+        if (KPT > 0) return reg[i];
+        return order_key(__ldg(score + i0 + i));
+    };
+
     uint32_t prefix = 0, pmask = 0, krem = static_cast<uint32_t>(k);
-    for (int pass = 0; pass < 4; ++pass) {
-        const int shift = 24 - 8 * pass;
-        for (int i = tid; i < kWarps * 256; i += kThreads) (&hist[0][0])[i] = 0;
+#pragma unroll 1
+    for (int pass = 0; pass < 3; ++pass) {
+        const int shift = pass == 0 ? 21 : (pass == 1 ? 10 : 0);
+        const uint32_t dmask = pass == 2 ? 0x3FFu : 0x7FFu;
+        for (int b = tid; b < kBins; b += kThreads) hist[b] = 0;
         __syncthreads();
-        for (int i = tid; i < n; i += kThreads) {
-            const uint32_t key = order_key(__ldg(score + i));
-            if ((key & pmask) == prefix) atomicAdd(&hist[warp][(key >> shift) & 255u], 1u);
+        if (KPT > 0) {
+#pragma unroll
+            for (int i = 0; i < (KPT > 0 ? KPT : 1); ++i) {
+                const uint32_t key = reg[i];
+                hist_add(hist, (key >> shift) & dmask, i < cnt && (key & pmask) == prefix);
+            }
+        } else {
+            for (int i = 0; i < per; ++i) {   // per is uniform; lanes past n are inactive
+                const uint32_t key = i < cnt ? key_at(i) : 0u;
+                hist_add(hist, (key >> shift) & dmask, i < cnt && (key & pmask) == prefix);
+            }
         }
         __syncthreads();
-        if (tid < 256) {
-            uint32_t c = 0;
-#pragma unroll 8
-            for (int w = 0; w < kWarps; ++w) c += hist[w][tid];
-            total[tid] = c;
-        }
-        __syncthreads();
-        if (warp == 0) {
-            // lane l scans bins 255-8l down to 248-8l; lanes in order cover bins high -> low
-            uint32_t cnt[8], local = 0;
-#pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                cnt[j] = total[255 - 8 * lane - j];
-                local += cnt[j];
-            }
-            uint32_t incl = local;
-#pragma unroll
-            for (int o = 1; o < 32; o *= 2) {
-                const uint32_t up = __shfl_up_sync(0xFFFFFFFFu, incl, o);
-                if (lane >= o) incl += up;
-            }
-            uint32_t above = incl - local;
-#pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                if (above < krem && above + cnt[j] >= krem) {
-                    s_digit = 255u - 8u * lane - j;
-                    s_krem = krem - above;
-                }
-                above += cnt[j];
+        // thread t holds bins 2047-2t and 2046-2t; an inclusive scan from the top
+        // finds the bin in which the k-th largest key falls
+        const uint32_t hi = hist[kBins - 1 - 2 * tid], lo = hist[kBins - 2 - 2 * tid];
+        const unsigned long long incl =
+            block_incl_scan<unsigned long long>(static_cast<unsigned long long>(hi + lo), wsum);
+        const unsigned long long above = incl - (hi + lo);
+        if (above < krem && incl >= krem) {
+            if (above + hi >= krem) {
+                s_digit = static_cast<uint32_t>(kBins - 1 - 2 * tid);
+                s_krem = krem - static_cast<uint32_t>(above);
+            } else {
+                s_digit = static_cast<uint32_t>(kBins - 2 - 2 * tid);
+                s_krem = krem - static_cast<uint32_t>(above) - hi;
             }
         }
         __syncthreads();
         prefix |= s_digit << shift;
-        pmask |= 0xFFu << shift;
+        pmask |= dmask << shift;
         krem = s_krem;
-        __syncthreads();
+        __syncthreads();   // s_digit / wsum are rewritten by the next pass
     }
     // prefix = K*; krem = how many keys equal to K* are selected (lowest indices first)
     const uint32_t kstar = prefix;
-    uint32_t run_gt = 0, run_eq = 0;
-    const uint32_t lt_mask = (1u << lane) - 1u;
-    for (int base = 0; base < n; base += kThreads) {
-        const int i = base + tid;
-        const uint32_t key = (i < n) ? order_key(__ldg(score + i)) : 0u;
-        const bool gt = (i < n) && key > kstar;
-        const bool eq = (i < n) && key == kstar;
-        const uint32_t bg = __ballot_sync(0xFFFFFFFFu, gt);
-        const uint32_t be = __ballot_sync(0xFFFFFFFFu, eq);
-        if (lane == 0) {
-            wcnt[warp][0] = __popc(bg);
-            wcnt[warp][1] = __popc(be);
+    uint32_t gt = 0, eq = 0;
+    if (KPT > 0) {
+#pragma unroll
+        for (int i = 0; i < (KPT > 0 ? KPT : 1); ++i) {
+            gt += (i < cnt && reg[i] > kstar);
+            eq += (i < cnt && reg[i] == kstar);
         }
-        __syncthreads();
-        uint32_t pre_g = 0, pre_e = 0, tot_g = 0, tot_e = 0;
-        for (int w = 0; w < kWarps; ++w) {   // broadcast reads; 32 entries
-            const uint32_t cg = wcnt[w][0], ce = wcnt[w][1];
-            if (w < warp) { pre_g += cg; pre_e += ce; }
-            tot_g += cg;
-            tot_e += ce;
+    } else {
+        for (int i = 0; i < cnt; ++i) {
+            const uint32_t key = key_at(i);
+            gt += key > kstar;
+            eq += key == kstar;
         }
-        const uint32_t eq_before = run_eq + pre_e + __popc(be & lt_mask);
-        const uint32_t gt_before = run_gt + pre_g + __popc(bg & lt_mask);
-        if (gt || (eq && eq_before < krem)) {
-            const uint32_t pos = gt_before + min(eq_before, krem);
-            out[pos] = idx_base + i;
+    }
+    const unsigned long long mine = (static_cast<unsigned long long>(gt) << 32) | eq;
+    const unsigned long long before = block_incl_scan<unsigned long long>(mine, wsum) - mine;
+    const uint32_t gt_before = static_cast<uint32_t>(before >> 32);
+    uint32_t eq_seen = static_cast<uint32_t>(before & 0xFFFFFFFFu);
+    uint32_t pos = gt_before + min(eq_seen, krem);
+    if (KPT > 0) {
+#pragma unroll
+        for (int i = 0; i < (KPT > 0 ? KPT : 1); ++i) {
+            const uint32_t key = reg[i];
+            if (i < cnt && (key > kstar || (key == kstar && eq_seen++ < krem)))
+                out[pos++] = idx_base + i0 + i;
         }
-        run_gt += tot_g;
-        run_eq += tot_e;
-        __syncthreads();
+    } else {
+        for (int i = 0; i < cnt; ++i) {
+            const uint32_t key = key_at(i);
+            if (key > kstar || (key == kstar && eq_seen++ < krem)) out[pos++] = idx_base + i0 + i;
+        }
     }
 }
 
@@ -120,8 +171,15 @@ select_kernel(const uint32_t *__restrict__ score, int n, int k, int idx_base, in
 cudaError_t launch_select(const float *score, int n, int k, int idx_base, int *out,
                           cudaStream_t s) {
     if (k == 0 || n == 0) return cudaSuccess;
-    select_kernel<<<1, kThreads, 0, s>>>(reinterpret_cast<const uint32_t *>(score), n, k, idx_base,
-                                         out);
+    const uint32_t *keys = reinterpret_cast<const uint32_t *>(score);
+    const int per = (n + kThreads - 1) / kThreads;
+    if (per <= 4) {
+        select_kernel<4><<<1, kThreads, 0, s>>>(keys, n, k, idx_base, 4, out);
+    } else if (per <= kRegKeys) {
+        select_kernel<kRegKeys><<<1, kThreads, 0, s>>>(keys, n, k, idx_base, kRegKeys, out);
+    } else {
+        select_kernel<0><<<1, kThreads, 0, s>>>(keys, n, k, idx_base, per, out);
+    }
     return cudaGetLastError();
 }
 

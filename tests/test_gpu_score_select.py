@@ -61,7 +61,7 @@ def _check_select(cs, vals, k, base):
     assert np.array_equal(got.cpu().numpy(), exp)
 
 
-@pytest.mark.parametrize("n", [1, 7, 1023, 1024, 1025, 3072, 64512, 100003])
+@pytest.mark.parametrize("n", [1, 7, 1023, 1024, 1025, 3072, 4096, 4097, 15360, 16384, 16385, 64512, 100003])
 def test_select_matches_oracle(cslib, n):
     rng = np.random.default_rng(n)
     cont = (rng.lognormal(0, 1.5, n) * 256).astype(np.float32)
