@@ -157,6 +157,28 @@ cs_status cs_repair_attention(const void *q, const void *k, const void *v, void 
                               const int32_t *qpos, float scale, void *stream);
 
 /*
+ * Scatter-back of repaired rows (Sec. 2: the recomputed tokens' fresh keys and
+ * values replace their stored ones in the composed cache before each layer's
+ * attention).  For every layer l < n_layers and row r < n_rows:
+ *   cache[l][idx[r]][:] = rows[l][r][:]          (row_elems elements per token)
+ *
+ *   cache      [n_layers][T][row_elems], layer stride cache_layer_stride
+ *              (elements, >= T*row_elems), device memory, written in place
+ *   rows       [n_layers][n_rows][row_elems], layer stride rows_layer_stride
+ *              (>= n_rows*row_elems), device memory, read only; must not overlap cache
+ *   idx        int32 [n_rows], device memory, distinct destination tokens;
+ *              0 <= idx[r] < T is checked on the device: a row outside is
+ *              skipped and cs_sync_status then returns CS_ERR_DEVICE_ARG
+ *   row_elems  elements of one token row, e.g. n_kv_heads * head_dim; the row
+ *              bytes, both layer strides in bytes and both pointers must be
+ *              multiples of 16
+ * Call once for the keys and once for the values.  Asynchronous on `stream`.
+ */
+cs_status cs_scatter_rows(void *cache, const void *rows, cs_dtype dtype, int n_layers, int T,
+                          int64_t cache_layer_stride, int n_rows, int64_t rows_layer_stride,
+                          int row_elems, const int32_t *idx, void *stream);
+
+/*
  * Waits for `stream`, then reports and clears the device status word of the
  * current device: CS_ERR_TIMEOUT or CS_ERR_DEVICE_ARG if a kernel recorded one
  * since the last call, CS_ERR_CUDA if the stream reported an error, else CS_OK.

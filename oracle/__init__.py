@@ -11,6 +11,7 @@ Plain, slow numpy code, written from the paper (arxiv 2607.19547, ChronoStitch):
   * score_f64 / score_f32_canonical   Eq. 5   delta_t = ||k_fresh - k_stored||_2 (squared)
   * select_topk         Sec. 2     top-rho later-chunk tokens
   * repair_attention    Eq. 1, Sec. 2   causal attention of the selected rows
+  * scatter_rows        Sec. 2     fresh rows of the repaired tokens written into the cache
 Floating point is fp64, with two deliberate exceptions where a float decides
 an integer and both sides must take that decision in the same precision:
   * stored results are rounded to the storage dtype (round_to_bf16 / fp32 RN);
@@ -246,6 +247,19 @@ def select_topk(score_f32, k: int, idx_base: int = 0) -> np.ndarray:
 # ----------------------------------------------------------------------------
 # Eq. 1 + Sec. 2: repair attention of the selected rows
 # ----------------------------------------------------------------------------
+
+
+def scatter_rows(cache, rows, idx) -> np.ndarray:
+    """Scatter-back (Sec. 2): the recomputed tokens' fresh keys/values replace their stored rows.
+
+    cache [L, T, ...], rows [L, n, ...], idx [n] distinct token indices in [0, T).
+    Returns a new array with cache[l, idx[r]] = rows[l, r] for every layer and row.
+    """
+    out = np.array(cache, copy=True)
+    idx = np.asarray(idx, dtype=np.int64)
+    for r, t in enumerate(idx):
+        out[:, t] = rows[:, r]
+    return out
 
 
 def repair_attention(q, k, v, qpos, scale=None, rows=None, layers=None):

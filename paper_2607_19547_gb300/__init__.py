@@ -8,6 +8,8 @@ kernel launch in the library:
   cs_score_deviation   Eq. 5  squared deviation of fresh vs re-based layer-1 keys
   cs_select_topk       Sec. 2 top-rho later-chunk tokens, lower index wins ties
   cs_repair_attention  Eq. 1  causal GQA attention of the selected rows over the cache
+and the scatter-back of the repaired rows' fresh keys and values:
+  cs_scatter_rows      Sec. 2 cache[l, idx[r]] = rows[l, r]
 
 This module only marshals torch tensors (device memory and streams) into the
 C calls and raises CsError on a non-OK status.  There is no CPU path: if the
@@ -49,6 +51,8 @@ _SIGS = {
     "cs_select_topk": (ctypes.c_int, [_vp, _i32, _i32, ctypes.c_int32, _vp, _vp]),
     "cs_repair_attention": (ctypes.c_int, [_vp, _vp, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _i32,
                                            _i32, _i32, _i64, _vp, _f32, _vp]),
+    "cs_scatter_rows": (ctypes.c_int, [_vp, _vp, _i32, _i32, _i32, _i64, _i32, _i64, _i32, _vp,
+                                       _vp]),
     "cs_sync_status": (ctypes.c_int, [_vp]),
     "cs_debug_wait_timeout": (ctypes.c_int, [ctypes.c_uint32, _vp]),
     "cs_status_string": (ctypes.c_char_p, [ctypes.c_int]),
@@ -221,6 +225,33 @@ def cs_repair_attention(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, qpos:
     return out
 
 
+def cs_scatter_rows(cache: torch.Tensor, rows: torch.Tensor, idx: torch.Tensor, *,
+                    stream=None) -> torch.Tensor:
+    """Sec. 2 scatter-back: cache[l, idx[r]] = rows[l, r] for cache [L, T, ...], rows [L, n, ...].
+
+    idx is int32 [n] of distinct tokens.  The cache is written in place and returned."""
+    _need_cuda(cache, rows, idx)
+    if cache.dim() < 2 or rows.dim() != cache.dim() or rows.shape[0] != cache.shape[0] or \
+            rows.shape[2:] != cache.shape[2:] or rows.dtype != cache.dtype:
+        raise ValueError("rows must be [L, n, ...] matching cache [L, T, ...] past the second dim")
+    _inner_contiguous(cache, "cache")
+    _inner_contiguous(rows, "rows")
+    if idx.dtype != torch.int32 or idx.dim() != 1 or idx.numel() != rows.shape[1] or \
+            not idx.is_contiguous():
+        raise ValueError("idx must be contiguous int32 [n]")
+    L, T = cache.shape[0], cache.shape[1]
+    n = rows.shape[1]
+    row_elems = 1
+    for d in cache.shape[2:]:
+        row_elems *= d
+    cs_stride = cache.stride(0) if L > 1 else T * row_elems
+    rs_stride = rows.stride(0) if L > 1 else n * row_elems
+    st = lib().cs_scatter_rows(cache.data_ptr(), rows.data_ptr(), _dtype_code(cache), L, T, cs_stride,
+                               n, rs_stride, row_elems, idx.data_ptr(), _stream(stream))
+    _check(st, "cs_scatter_rows")
+    return cache
+
+
 def cs_sync_status(stream=None) -> None:
     """Waits for the stream and raises CsError if a kernel recorded a device-side error."""
     _check(lib().cs_sync_status(_stream(stream)), "cs_sync_status")
@@ -232,5 +263,5 @@ def cs_debug_wait_timeout(limit_us: int, stream=None) -> None:
 
 
 __all__ = ["cs_rebase_keys", "cs_score_deviation", "cs_select_topk", "cs_repair_attention",
-           "cs_sync_status", "cs_debug_wait_timeout", "cs_status_string", "cs_last_error_detail",
+           "cs_scatter_rows", "cs_sync_status", "cs_debug_wait_timeout", "cs_status_string", "cs_last_error_detail",
            "cs_abi_version", "CsError", "lib", "LIB_PATH"]

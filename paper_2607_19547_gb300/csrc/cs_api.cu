@@ -198,6 +198,43 @@ cs_status cs_select_topk(const float *score, int n, int k, int32_t idx_base, int
     return CS_OK;
 }
 
+cs_status cs_scatter_rows(void *cache, const void *rows, cs_dtype dtype, int n_layers, int T,
+                          int64_t cache_layer_stride, int n_rows, int64_t rows_layer_stride,
+                          int row_elems, const int32_t *idx, void *stream) {
+    if (dtype != CS_DTYPE_F32 && dtype != CS_DTYPE_BF16) return fail(CS_ERR_INVALID_ARG, "dtype");
+    if (n_layers < 0 || T < 0 || n_rows < 0 || row_elems <= 0)
+        return fail(CS_ERR_INVALID_ARG, "negative size or non-positive row_elems");
+    const long long esz = dtype == CS_DTYPE_BF16 ? 2 : 4;
+    if ((row_elems * esz) % 16)
+        return fail(CS_ERR_UNSUPPORTED, "row bytes %lld not a multiple of 16", row_elems * esz);
+    if (cache_layer_stride < static_cast<long long>(T) * row_elems)
+        return fail(CS_ERR_INVALID_ARG, "cache_layer_stride < T*row_elems");
+    if (rows_layer_stride < static_cast<long long>(n_rows) * row_elems)
+        return fail(CS_ERR_INVALID_ARG, "rows_layer_stride < n_rows*row_elems");
+    if (n_layers == 0 || n_rows == 0) return CS_OK;
+    if (T == 0) return fail(CS_ERR_INVALID_ARG, "rows to scatter into an empty cache");
+    if (cache == nullptr || rows == nullptr || idx == nullptr)
+        return fail(CS_ERR_INVALID_ARG, "NULL pointer");
+    if (!aligned16(cache) || !aligned16(rows) || (cache_layer_stride * esz) % 16 ||
+        (rows_layer_stride * esz) % 16)
+        return fail(CS_ERR_INVALID_ARG, "cache, rows and layer strides must be 16-byte aligned");
+    {
+        const char *c = static_cast<const char *>(cache);
+        const char *r = static_cast<const char *>(rows);
+        const long long cspan = ((n_layers - 1) * cache_layer_stride + static_cast<long long>(T) * row_elems) * esz;
+        const long long rspan = ((n_layers - 1) * rows_layer_stride + static_cast<long long>(n_rows) * row_elems) * esz;
+        if (c < r + rspan && r < c + cspan) return fail(CS_ERR_INVALID_ARG, "rows overlap the cache");
+    }
+    unsigned int *status = status_word();
+    if (status == nullptr) return CS_ERR_CUDA;
+    const long long row16 = row_elems * esz / 16;
+    const cudaError_t e = launch_scatter(cache, rows, n_layers, T, cache_layer_stride * esz / 16, n_rows,
+                                         rows_layer_stride * esz / 16, static_cast<int>(row16), idx,
+                                         status, as_stream(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "scatter launch");
+    return CS_OK;
+}
+
 cs_status cs_repair_attention(const void *q, const void *k, const void *v, void *o, float *lse,
                               cs_dtype dtype, int n_layers, int M, int T, int n_q_heads,
                               int n_kv_heads, int head_dim, int64_t kv_layer_stride,

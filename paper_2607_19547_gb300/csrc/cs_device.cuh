@@ -16,6 +16,7 @@ enum : unsigned int {
     kSiteAttnSoftmax = 3,
     kSiteAttnQpos = 4,
     kSiteDebugWait = 5,
+    kSiteScatter = 6,
 };
 
 // Records the first error on this device: word[0] = code, word[1] = site, word[2] = detail.

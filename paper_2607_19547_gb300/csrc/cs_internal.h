@@ -40,6 +40,11 @@ struct RebaseArgs {
 };
 cudaError_t launch_rebase(const RebaseArgs &a, cs_dtype dt, cudaStream_t s);
 
+// ---- scatter-back (scatter.cu) -----------------------------------------------
+cudaError_t launch_scatter(void *cache, const void *rows, int n_layers, int T, long long cache_stride16,
+                           int n_rows, long long rows_stride16, int row16, const int *idx,
+                           unsigned int *status, cudaStream_t s);
+
 // ---- score (score.cu) --------------------------------------------------------
 cudaError_t launch_score(const void *fresh, const void *cached, cs_dtype dt, int n, int E,
                          long long fresh_stride, long long cached_stride, float *out,

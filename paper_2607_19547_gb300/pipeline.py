@@ -9,6 +9,17 @@ and runs the four calls of the hot path in stream order:
   4. cs_repair_attention the k selected rows plus the S suffix rows over the cache (Eq. 1)
 Query tensors of the repaired rows and the fresh keys of the candidates come
 from the model (projections and a shallow recompute, outside this library).
+
+Options around the four calls:
+  * policy: "3axis" (Eq. 3, the method), "scalar1d" (every token re-based to the
+    scalar slot (i, i, i) of its sequence position, the 1-D re-index baseline of
+    Sec. 2 / Table 1) or "naive" (stored keys used as they are, no re-base);
+  * fresh_kv: the repaired rows' fresh keys and values [L, k, Hkv, D], written
+    into the cache at the selected positions (cs_scatter_rows) before the
+    attention, as the recompute does layer by layer (Sec. 2);
+  * shallow_recompute(): the attention part of the shallow recompute, every
+    candidate as a query row over the first layers (the 2 c_a |C| T term of
+    Eq. 6), run with the same attention kernel.
 """
 from __future__ import annotations
 
@@ -16,7 +27,10 @@ import dataclasses
 
 import torch
 
-from . import cs_rebase_keys, cs_repair_attention, cs_score_deviation, cs_select_topk
+from . import (cs_rebase_keys, cs_repair_attention, cs_scatter_rows, cs_score_deviation,
+               cs_select_topk)
+
+POLICIES = ("3axis", "scalar1d", "naive")
 
 
 @dataclasses.dataclass
@@ -50,18 +64,50 @@ class ComposedQuery:
         if s.suffix:
             self.qpos[s.k:] = torch.arange(s.T - s.suffix, s.T, dtype=torch.int32, device=device)
         self.out = torch.empty((s.n_layers, s.M, s.hq, s.head_dim), dtype=dtype, device=device)
+        self.device = device
+        self._scalar_targets = None
+        self._cand_pos = None
 
-    def step(self, k, v, q, k_fresh, pos_local, pos_global, stream=None):
+    def scalar_targets(self) -> torch.Tensor:
+        """int32 [T, 3] with row i = (i, i, i): the scalar re-index targets."""
+        if self._scalar_targets is None:
+            i = torch.arange(self.shape.T, dtype=torch.int32, device=self.device)
+            self._scalar_targets = torch.stack([i, i, i], dim=1).contiguous()
+        return self._scalar_targets
+
+    def step(self, k, v, q, k_fresh, pos_local, pos_global, stream=None, policy="3axis",
+             fresh_kv=None):
         """Runs the four calls on `stream`; returns (attention output, query positions).
 
-        k is re-based in place: after the call it is the composed cache."""
+        k is re-based in place: after the call it is the composed cache (with the
+        repaired rows' fresh keys and values when fresh_kv is given)."""
         s = self.shape
-        cs_rebase_keys(k, pos_local, pos_global, theta=s.theta, sections=s.sections, stream=stream)
+        if policy not in POLICIES:
+            raise ValueError(f"policy must be one of {POLICIES}")
+        if policy == "3axis":
+            cs_rebase_keys(k, pos_local, pos_global, theta=s.theta, sections=s.sections, stream=stream)
+        elif policy == "scalar1d":
+            cs_rebase_keys(k, pos_local, self.scalar_targets(), theta=s.theta, sections=s.sections,
+                           stream=stream)
         cached = k[s.score_layer, s.cand0:s.cand0 + s.n_cand]
         cs_score_deviation(k_fresh, cached, out=self.score, stream=stream)
         cs_select_topk(self.score, s.k, s.cand0, out=self.qpos[:s.k], stream=stream)
+        if fresh_kv is not None:
+            k_rows, v_rows = fresh_kv
+            cs_scatter_rows(k, k_rows, self.qpos[:s.k], stream=stream)
+            cs_scatter_rows(v, v_rows, self.qpos[:s.k], stream=stream)
         cs_repair_attention(q, k, v, self.qpos, out=self.out, stream=stream)
         return self.out, self.qpos
+
+    def shallow_recompute(self, q_cand, k, v, stream=None, out=None):
+        """Attention of every candidate token over the composed cache for the first
+        q_cand.shape[0] layers (q_cand [layers, n_cand, Hq, D]); returns [layers, n_cand, Hq, D]."""
+        s = self.shape
+        if self._cand_pos is None:
+            self._cand_pos = torch.arange(s.cand0, s.cand0 + s.n_cand, dtype=torch.int32,
+                                          device=self.device)
+        nl = q_cand.shape[0]
+        return cs_repair_attention(q_cand, k[:nl], v[:nl], self._cand_pos, out=out, stream=stream)
 
 
 def compose_from_host(query: ComposedQuery, host: dict, dev: dict, out_host: dict, stream=None):

@@ -146,3 +146,27 @@ def test_python_binding_refuses_cpu_tensors(cslib):
     pos = torch.zeros(4, 3, dtype=torch.int32)
     with pytest.raises(ValueError):
         cslib.cs_rebase_keys(k, pos, pos)
+
+
+def test_scatter_rejects_bad_arguments(cslib):
+    L = cslib.lib()
+
+    def call(**kw):
+        a = dict(cache=FAKE, rows=FAKE + (1 << 24), dt=1, L=2, T=10, cst=10 * 256, n=3, rst=3 * 256,
+                 re=256, idx=FAKE)
+        a.update(kw)
+        return L.cs_scatter_rows(a["cache"], a["rows"], a["dt"], a["L"], a["T"], a["cst"], a["n"],
+                                 a["rst"], a["re"], a["idx"], None)
+
+    assert call(dt=7) == cslib.CS_ERR_INVALID_ARG
+    assert call(n=-1) == cslib.CS_ERR_INVALID_ARG
+    assert call(re=0) == cslib.CS_ERR_INVALID_ARG
+    assert call(re=5) == cslib.CS_ERR_UNSUPPORTED            # 10-byte rows
+    assert call(cst=100) == cslib.CS_ERR_INVALID_ARG         # stride < T * row
+    assert call(rst=100) == cslib.CS_ERR_INVALID_ARG
+    assert call(idx=None) == cslib.CS_ERR_INVALID_ARG
+    assert call(cache=FAKE + 8) == cslib.CS_ERR_INVALID_ARG  # misaligned
+    assert call(rows=FAKE + 512) == cslib.CS_ERR_INVALID_ARG  # overlaps the cache
+    assert call(T=0, cst=0) == cslib.CS_ERR_INVALID_ARG
+    assert call(n=0, rows=None, idx=None) == cslib.CS_OK
+    assert call(L=0) == cslib.CS_OK

@@ -386,3 +386,24 @@ def test_attention_invariant_under_common_shift():
     qs = O.rebase_f64(q, p[qrows], p[qrows] + shift)
     o2, _ = O.repair_attention(qs, ks, v, qrows)
     np.testing.assert_allclose(o2, o1, atol=1e-11)
+
+
+def test_scatter_rows_by_definition():
+    """Scatter-back (Sec. 2): a hand-built case, the identity when the rows already are the
+    cache's, and every untouched row bit-identical."""
+    cache = np.arange(2 * 5 * 3, dtype=np.float64).reshape(2, 5, 3)
+    rows = -np.arange(1, 2 * 2 * 3 + 1, dtype=np.float64).reshape(2, 2, 3)
+    out = O.scatter_rows(cache, rows, [3, 0])
+    exp = cache.copy()
+    exp[0, 3], exp[1, 3] = [-1, -2, -3], [-7, -8, -9]
+    exp[0, 0], exp[1, 0] = [-4, -5, -6], [-10, -11, -12]
+    assert np.array_equal(out, exp)
+    assert np.array_equal(cache, np.arange(30, dtype=np.float64).reshape(2, 5, 3))   # input kept
+    rng = np.random.default_rng(3)
+    big = rng.standard_normal((3, 40, 2, 8))
+    idx = np.sort(rng.choice(40, 11, replace=False))
+    assert np.array_equal(O.scatter_rows(big, big[:, idx], idx), big)
+    fresh = rng.standard_normal((3, 11, 2, 8))
+    got = O.scatter_rows(big, fresh, idx)
+    keep = np.setdiff1d(np.arange(40), idx)
+    assert np.array_equal(got[:, keep], big[:, keep]) and np.array_equal(got[:, idx], fresh)
