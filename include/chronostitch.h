@@ -116,6 +116,29 @@ cs_status cs_score_deviation(const void *k_fresh, const void *k_cached, cs_dtype
                              int64_t cached_row_stride, float *score_out, void *stream);
 
 /*
+ * Steps 1 and 2 in one call (Eq. 3 then Eq. 5 at the score layer, Sec. 2):
+ * exactly cs_rebase_keys(...) followed by
+ *   cs_score_deviation(k_fresh, k_out + (score_layer*layer_stride + cand0*E),
+ *                      dtype, n_cand, n_kv_heads, head_dim, fresh_row_stride, E,
+ *                      score_out)              with E = n_kv_heads*head_dim,
+ * bit for bit, where the candidates are tokens [cand0, cand0 + n_cand) of the
+ * cache.  For bf16 with n_kv_heads 1, 2 or 4 it is one kernel launch: the
+ * re-base computes the scores of the rows it has just re-based; otherwise two.
+ *
+ *   0 <= score_layer < n_layers (when n_cand > 0);  0 <= cand0,  cand0 + n_cand <= T
+ *   k_fresh    row c (token cand0 + c) at k_fresh + c*fresh_row_stride, E elements,
+ *              device memory, 16-byte aligned rows, not overlapping k_out
+ *   score_out  fp32 [n_cand], device memory
+ * Other arguments and errors as for cs_rebase_keys and cs_score_deviation.
+ */
+cs_status cs_rebase_and_score(const void *k_in, void *k_out, cs_dtype dtype, int n_layers,
+                              int64_t layer_stride, int T, int n_kv_heads, int head_dim,
+                              const int32_t *pos_local, const int32_t *pos_global,
+                              const cs_rope_cfg *rope, int score_layer, int cand0, int n_cand,
+                              const void *k_fresh, int64_t fresh_row_stride, float *score_out,
+                              void *stream);
+
+/*
  * Step 3 - top-rho selection (Sec. 2).
  *
  * Writes the k candidates with the largest score as ascending global indices

@@ -8,7 +8,8 @@ kernel launch in the library:
   cs_score_deviation   Eq. 5  squared deviation of fresh vs re-based layer-1 keys
   cs_select_topk       Sec. 2 top-rho later-chunk tokens, lower index wins ties
   cs_repair_attention  Eq. 1  causal GQA attention of the selected rows over the cache
-and the scatter-back of the repaired rows' fresh keys and values:
+plus cs_rebase_and_score (steps 1 and 2 in one launch where possible) and the
+scatter-back of the repaired rows' fresh keys and values:
   cs_scatter_rows      Sec. 2 cache[l, idx[r]] = rows[l, r]
 
 This module only marshals torch tensors (device memory and streams) into the
@@ -48,6 +49,9 @@ _SIGS = {
     "cs_rebase_keys": (ctypes.c_int, [_vp, _vp, _i32, _i32, _i64, _i32, _i32, _i32, _vp, _vp,
                                       ctypes.POINTER(_RopeCfg), _vp]),
     "cs_score_deviation": (ctypes.c_int, [_vp, _vp, _i32, _i32, _i32, _i32, _i64, _i64, _vp, _vp]),
+    "cs_rebase_and_score": (ctypes.c_int, [_vp, _vp, _i32, _i32, _i64, _i32, _i32, _i32, _vp, _vp,
+                                           ctypes.POINTER(_RopeCfg), _i32, _i32, _i32, _vp, _i64,
+                                           _vp, _vp]),
     "cs_select_topk": (ctypes.c_int, [_vp, _i32, _i32, ctypes.c_int32, _vp, _vp]),
     "cs_repair_attention": (ctypes.c_int, [_vp, _vp, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _i32,
                                            _i32, _i32, _i64, _vp, _f32, _vp]),
@@ -149,6 +153,47 @@ def cs_rebase_keys(k: torch.Tensor, pos_local: torch.Tensor, pos_global: torch.T
                               ctypes.byref(cfg), _stream(stream))
     _check(st, "cs_rebase_keys")
     return out
+
+
+def cs_rebase_and_score(k: torch.Tensor, pos_local: torch.Tensor, pos_global: torch.Tensor,
+                        k_fresh: torch.Tensor, score_layer: int, cand0: int, *,
+                        score_out: torch.Tensor | None = None, k_out: torch.Tensor | None = None,
+                        theta: float = 1e6, sections=(16, 24, 24), stream=None):
+    """Eq. 3 then Eq. 5: re-base k [L, T, Hkv, D] (in place unless k_out) and score the
+    n = k_fresh.shape[0] candidate tokens [cand0, cand0 + n) at layer score_layer against
+    k_fresh [n, Hkv, D] (rows may be strided).  One launch where the library can fuse them.
+    Returns (re-based keys, fp32 scores [n])."""
+    _need_cuda(k, pos_local, pos_global, k_fresh)
+    if k.dim() != 4:
+        raise ValueError("k must be [L, T, Hkv, D]")
+    _inner_contiguous(k, "k")
+    out = k if k_out is None else k_out
+    if out is not k:
+        _need_cuda(out)
+        if out.shape != k.shape or out.dtype != k.dtype or out.stride() != k.stride():
+            raise ValueError("k_out must match k in shape, dtype and strides")
+    for p in (pos_local, pos_global):
+        if p.dtype != torch.int32 or not p.is_contiguous() or p.shape != (k.shape[1], 3):
+            raise ValueError("coordinates must be contiguous int32 [T, 3]")
+    L, T, H, D = k.shape
+    if k_fresh.dim() != 3 or k_fresh.shape[1:] != (H, D) or k_fresh.dtype != k.dtype:
+        raise ValueError("k_fresh must be [n, Hkv, D] of the keys' dtype")
+    _inner_contiguous(k_fresh, "k_fresh")
+    n = k_fresh.shape[0]
+    if score_out is None:
+        score_out = torch.empty(n, dtype=torch.float32, device=k.device)
+    _need_cuda(score_out)
+    if score_out.dtype != torch.float32 or score_out.numel() < n or not score_out.is_contiguous():
+        raise ValueError("score_out must be contiguous fp32 with n elements")
+    cfg = _RopeCfg(float(theta), (ctypes.c_int32 * 3)(*[int(s) for s in sections]))
+    fs = k_fresh.stride(0) if n > 1 else H * D
+    st = lib().cs_rebase_and_score(k.data_ptr(), out.data_ptr(), _dtype_code(k), L,
+                                   k.stride(0) if L > 1 else T * H * D, T, H, D,
+                                   pos_local.data_ptr(), pos_global.data_ptr(), ctypes.byref(cfg),
+                                   int(score_layer), int(cand0), n, k_fresh.data_ptr(), fs,
+                                   score_out.data_ptr(), _stream(stream))
+    _check(st, "cs_rebase_and_score")
+    return out, score_out
 
 
 def cs_score_deviation(k_fresh: torch.Tensor, k_cached: torch.Tensor, *,
@@ -262,6 +307,6 @@ def cs_debug_wait_timeout(limit_us: int, stream=None) -> None:
     _check(lib().cs_debug_wait_timeout(int(limit_us), _stream(stream)), "cs_debug_wait_timeout")
 
 
-__all__ = ["cs_rebase_keys", "cs_score_deviation", "cs_select_topk", "cs_repair_attention",
+__all__ = ["cs_rebase_keys", "cs_rebase_and_score", "cs_score_deviation", "cs_select_topk", "cs_repair_attention",
            "cs_scatter_rows", "cs_sync_status", "cs_debug_wait_timeout", "cs_status_string", "cs_last_error_detail",
            "cs_abi_version", "CsError", "lib", "LIB_PATH"]

@@ -102,10 +102,20 @@ const char *cs_status_string(cs_status s) {
 
 const char *cs_last_error_detail(void) { return t_detail; }
 
-cs_status cs_rebase_keys(const void *k_in, void *k_out, cs_dtype dtype, int n_layers,
-                         int64_t layer_stride, int T, int n_kv_heads, int head_dim,
-                         const int32_t *pos_local, const int32_t *pos_global,
-                         const cs_rope_cfg *rope, void *stream) {
+namespace {
+
+// The layer-`score_layer` score requested together with a re-base.
+struct ScoreRequest {
+    int score_layer, cand0, n_cand;
+    const void *fresh;
+    long long fresh_stride;
+    float *score_out;
+};
+
+cs_status rebase_impl(const void *k_in, void *k_out, cs_dtype dtype, int n_layers,
+                      int64_t layer_stride, int T, int n_kv_heads, int head_dim,
+                      const int32_t *pos_local, const int32_t *pos_global, const cs_rope_cfg *rope,
+                      const ScoreRequest *sc, void *stream) {
     if (dtype != CS_DTYPE_F32 && dtype != CS_DTYPE_BF16) return fail(CS_ERR_INVALID_ARG, "dtype");
     if (n_layers < 0 || T < 0 || n_kv_heads <= 0 || head_dim <= 0)
         return fail(CS_ERR_INVALID_ARG, "negative size or non-positive head count/dim");
@@ -127,13 +137,27 @@ cs_status cs_rebase_keys(const void *k_in, void *k_out, cs_dtype dtype, int n_la
     if (layer_stride < static_cast<long long>(T) * row)
         return fail(CS_ERR_INVALID_ARG, "layer_stride %lld < T*n_kv_heads*head_dim",
                     static_cast<long long>(layer_stride));
+    const long long esz = dtype == CS_DTYPE_BF16 ? 2 : 4;
+    const bool scoring = sc != nullptr && sc->n_cand > 0;
+    if (sc != nullptr) {
+        if (sc->n_cand < 0 || sc->cand0 < 0 || static_cast<long long>(sc->cand0) + sc->n_cand > T)
+            return fail(CS_ERR_INVALID_ARG, "candidates [cand0, cand0 + n_cand) must lie in [0, T)");
+        if (scoring && (sc->score_layer < 0 || sc->score_layer >= n_layers))
+            return fail(CS_ERR_INVALID_ARG, "score_layer %d outside [0, %d)", sc->score_layer, n_layers);
+        if (row > 2048) return fail(CS_ERR_UNSUPPORTED, "row of %lld elements > 2048", row);
+        if (sc->fresh_stride < row)
+            return fail(CS_ERR_INVALID_ARG, "fresh row stride shorter than n_kv_heads*head_dim");
+        if (scoring && (sc->fresh == nullptr || sc->score_out == nullptr))
+            return fail(CS_ERR_INVALID_ARG, "NULL fresh keys or score output");
+        if (scoring && (!aligned16(sc->fresh) || (sc->fresh_stride * esz) % 16))
+            return fail(CS_ERR_INVALID_ARG, "fresh rows must start 16-byte aligned");
+    }
     if (n_layers == 0 || T == 0) return CS_OK;
     if (k_in == nullptr || k_out == nullptr || pos_local == nullptr || pos_global == nullptr)
         return fail(CS_ERR_INVALID_ARG, "NULL tensor pointer");
-    if (!aligned16(k_in) || !aligned16(k_out) || (layer_stride * (dtype == CS_DTYPE_BF16 ? 2 : 4)) % 16)
+    if (!aligned16(k_in) || !aligned16(k_out) || (layer_stride * esz) % 16)
         return fail(CS_ERR_INVALID_ARG, "keys must be 16-byte aligned (pointers and layer stride)");
     if (k_in != k_out) {
-        const long long esz = dtype == CS_DTYPE_BF16 ? 2 : 4;
         const long long span = ((n_layers - 1) * layer_stride + T * row) * esz;
         const char *a = static_cast<const char *>(k_in);
         const char *b = static_cast<const char *>(k_out);
@@ -156,9 +180,47 @@ cs_status cs_rebase_keys(const void *k_in, void *k_out, cs_dtype dtype, int n_la
         for (int c = 0; c < rope->sections[a]; ++c, ++i) args.axis[i] = static_cast<unsigned char>(a);
     for (i = 0; i < head_dim / 2; ++i)
         args.turn_step[i] = turn_step(std::pow(rope->theta, -(2.0 * i) / head_dim));
-    const cudaError_t e = launch_rebase(args, dtype, as_stream(stream));
+    if (scoring) {
+        args.fresh = sc->fresh;
+        args.fresh_stride = sc->fresh_stride;
+        args.score_out = sc->score_out;
+        args.score_layer = sc->score_layer;
+        args.cand0 = sc->cand0;
+        args.n_cand = sc->n_cand;
+        if (!rebase_fuses_score(args, dtype)) args.score_out = nullptr;   // scored below
+    }
+    cudaError_t e = launch_rebase(args, dtype, as_stream(stream));
     if (e != cudaSuccess) return cuda_fail(e, "rebase launch");
+    if (scoring && args.score_out == nullptr) {
+        const char *cached = static_cast<const char *>(k_out) +
+                             (static_cast<long long>(sc->score_layer) * layer_stride +
+                              static_cast<long long>(sc->cand0) * row) * esz;
+        e = launch_score(sc->fresh, cached, dtype, sc->n_cand, static_cast<int>(row), sc->fresh_stride,
+                         row, sc->score_out, as_stream(stream));
+        if (e != cudaSuccess) return cuda_fail(e, "score launch");
+    }
     return CS_OK;
+}
+
+}  // namespace
+
+cs_status cs_rebase_keys(const void *k_in, void *k_out, cs_dtype dtype, int n_layers,
+                         int64_t layer_stride, int T, int n_kv_heads, int head_dim,
+                         const int32_t *pos_local, const int32_t *pos_global,
+                         const cs_rope_cfg *rope, void *stream) {
+    return rebase_impl(k_in, k_out, dtype, n_layers, layer_stride, T, n_kv_heads, head_dim, pos_local,
+                       pos_global, rope, nullptr, stream);
+}
+
+cs_status cs_rebase_and_score(const void *k_in, void *k_out, cs_dtype dtype, int n_layers,
+                              int64_t layer_stride, int T, int n_kv_heads, int head_dim,
+                              const int32_t *pos_local, const int32_t *pos_global,
+                              const cs_rope_cfg *rope, int score_layer, int cand0, int n_cand,
+                              const void *k_fresh, int64_t fresh_row_stride, float *score_out,
+                              void *stream) {
+    const ScoreRequest sc{score_layer, cand0, n_cand, k_fresh, fresh_row_stride, score_out};
+    return rebase_impl(k_in, k_out, dtype, n_layers, layer_stride, T, n_kv_heads, head_dim, pos_local,
+                       pos_global, rope, &sc, stream);
 }
 
 cs_status cs_score_deviation(const void *k_fresh, const void *k_cached, cs_dtype dtype, int n,

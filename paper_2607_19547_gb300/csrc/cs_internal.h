@@ -37,7 +37,16 @@ struct RebaseArgs {
     unsigned long long turn_step[64];   // theta_i / (2 pi) in units of 2^-64 turns
     unsigned char axis[64];             // sigma(i)
     int in_place;
+    // fused score of layer score_layer (bf16, n_kv_heads 1, 2 or 4): when score_out
+    // is set, score_out[t - cand0] = Eq. 5 squared of fresh row t - cand0 against
+    // the re-based row t, for t in [cand0, cand0 + n_cand)
+    const void *fresh;
+    long long fresh_stride;             // elements between fresh rows
+    float *score_out;
+    int score_layer, cand0, n_cand;
 };
+// Whether launch_rebase computes the fused score itself for these arguments.
+bool rebase_fuses_score(const RebaseArgs &a, cs_dtype dt);
 cudaError_t launch_rebase(const RebaseArgs &a, cs_dtype dt, cudaStream_t s);
 
 // ---- scatter-back (scatter.cu) -----------------------------------------------

@@ -210,53 +210,28 @@ __device__ __forceinline__ bool rotate_slice(const uint4 &xv, const uint4 &yv, c
     return ok;
 }
 
-// bf16: 8 threads per 128-element row, each owning 8 frequency pairs (16 bytes
-// of the first half and the matching 16 bytes of the second half).  A CTA
-// takes a block of TB tokens (TB * n_kv_heads * 8 threads per layer "slot")
-// and walks every layer of its range, n_slots layers at a time, so the cos/sin
-// table of its tokens is built once and reused across layers.
-//   - each thread reads its own token's delta and issues its first load before
-//     the table is built, so DRAM latency overlaps the sincos evaluation;
-//   - the next layer's slice is loaded before the current one is rotated;
-//   - a slice with an uncertain rounding is not stored; its layer is recorded
-//     and, after the streaming loop, redone in double-float from the untouched
-//     input (keeping the rare slow path out of the hot loop).
-__global__ void __launch_bounds__(kThreads, 4) rebase_bf16_kernel(RebaseArgs a, int TB, int l_per_cta) {
-    __shared__ float4 tab[kMaxTokensBf16 * 64];
-    __shared__ int s_delta[kMaxTokensBf16][3];
-    const int t0 = blockIdx.x * TB;
-    const int l0 = blockIdx.y * l_per_cta;
-    const int l1 = min(a.n_layers, l0 + l_per_cta);
-    const int slot_threads = TB * a.hkv * 8;
-    const int n_slots = kThreads / slot_threads;
-    const int slot = threadIdx.x / slot_threads;
-    const int loc = threadIdx.x - slot * slot_threads;
-    const int tb = loc / (a.hkv * 8);
-    const int h = (loc >> 3) % a.hkv;
-    const int pg = loc & 7;
-    const int t = t0 + tb;
-    const int lfirst = l0 + slot;
-    bool mine = (slot < n_slots) && (t < a.T) && (lfirst < l1);
-    bool moved = false;
-    if (mine) {
-        moved = ((a.pos_global[3 * t] - a.pos_local[3 * t]) |
-                 (a.pos_global[3 * t + 1] - a.pos_local[3 * t + 1]) |
-                 (a.pos_global[3 * t + 2] - a.pos_local[3 * t + 2])) != 0;
-        if (!moved && a.in_place) mine = false;
+// Eq. 5 block term of the canonical fp32 order: ((q0+q1)+(q2+q3))+((q4+q5)+(q6+q7)),
+// q = (fresh - cached)^2 rounded at every step, for one 16-byte word of each side.
+__device__ __forceinline__ float score_block8(uint4 fv, uint4 cv) {
+    const uint32_t fw[4] = {fv.x, fv.y, fv.z, fv.w};
+    const uint32_t cw[4] = {cv.x, cv.y, cv.z, cv.w};
+    float q[8];
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+        const float d0 = __fsub_rn(bf16_lo(fw[w]), bf16_lo(cw[w]));
+        const float d1 = __fsub_rn(bf16_hi(fw[w]), bf16_hi(cw[w]));
+        q[2 * w] = __fmul_rn(d0, d0);
+        q[2 * w + 1] = __fmul_rn(d1, d1);
     }
-    const int count = mine ? (l1 - lfirst + n_slots - 1) / n_slots : 0;
-    const __nv_bfloat16 *src = static_cast<const __nv_bfloat16 *>(a.k_in);
-    __nv_bfloat16 *dst = static_cast<__nv_bfloat16 *>(a.k_out);
-    const long long row0 = (static_cast<long long>(t) * a.hkv + h) * 128 + pg * 8;
-    const long long lstep = static_cast<long long>(n_slots) * a.layer_stride;
-    const long long obase = static_cast<long long>(lfirst) * a.layer_stride + row0;
-    uint4 xv = make_uint4(0, 0, 0, 0), yv = make_uint4(0, 0, 0, 0);
-    if (count > 0) {
-        xv = __ldcs(reinterpret_cast<const uint4 *>(src + obase));
-        yv = __ldcs(reinterpret_cast<const uint4 *>(src + obase + 64));
-    }
-    const bool moved_any = build_table(a, t0, TB, s_delta, tab);
-    if (count == 0) return;
+    return __fadd_rn(__fadd_rn(__fadd_rn(q[0], q[1]), __fadd_rn(q[2], q[3])),
+                     __fadd_rn(__fadd_rn(q[4], q[5]), __fadd_rn(q[6], q[7])));
+}
+
+// The streaming part of the bf16 kernel for one thread's slices (see the kernel below).
+__device__ __forceinline__ void stream_slices(const RebaseArgs &a, const __nv_bfloat16 *src,
+                                              __nv_bfloat16 *dst, long long obase, long long lstep,
+                                              int count, bool moved, bool moved_any, int tb, int pg,
+                                              const float4 *tab, uint4 xv, uint4 yv) {
     if (!moved) {   // out-of-place copy of an unmoved token
         for (int i = 0; i < count; ++i) {
             const long long o = obase + i * lstep;
@@ -307,6 +282,84 @@ __global__ void __launch_bounds__(kThreads, 4) rebase_bf16_kernel(RebaseArgs a, 
     }
 }
 
+// bf16: 8 threads per 128-element row, each owning 8 frequency pairs (16 bytes
+// of the first half and the matching 16 bytes of the second half).  A CTA
+// takes a block of TB tokens (TB * n_kv_heads * 8 threads per layer "slot")
+// and walks every layer of its range, n_slots layers at a time, so the cos/sin
+// table of its tokens is built once and reused across layers.
+//   - each thread reads its own token's delta and issues its first load before
+//     the table is built, so DRAM latency overlaps the sincos evaluation;
+//   - the next layer's slice is loaded before the current one is rotated;
+//   - a slice with an uncertain rounding is not stored; its layer is recorded
+//     and, after the streaming loop, redone in double-float from the untouched
+//     input (keeping the rare slow path out of the hot loop);
+//   - with the fused score, the slot that re-based layer score_layer reads its
+//     candidate rows back (its own stores) with the matching fresh rows and
+//     reduces each token's 16 * n_kv_heads block sums in the canonical halving
+//     order: token rows are adjacent lanes of one warp (8 lanes per head), so
+//     strides of 16 and more blocks are lane offsets of 8 and 16, the stride of
+//     8 blocks stays inside a thread (its two halves), and 4, 2, 1 are lane
+//     offsets again.
+__global__ void __launch_bounds__(kThreads, 4) rebase_bf16_kernel(RebaseArgs a, int TB, int l_per_cta) {
+    __shared__ float4 tab[kMaxTokensBf16 * 64];
+    __shared__ int s_delta[kMaxTokensBf16][3];
+    const int t0 = blockIdx.x * TB;
+    const int l0 = blockIdx.y * l_per_cta;
+    const int l1 = min(a.n_layers, l0 + l_per_cta);
+    const int slot_threads = TB * a.hkv * 8;
+    const int n_slots = kThreads / slot_threads;
+    const int slot = threadIdx.x / slot_threads;
+    const int loc = threadIdx.x - slot * slot_threads;
+    const int tb = loc / (a.hkv * 8);
+    const int h = (loc >> 3) % a.hkv;
+    const int pg = loc & 7;
+    const int t = t0 + tb;
+    const int lfirst = l0 + slot;
+    bool mine = (slot < n_slots) && (t < a.T) && (lfirst < l1);
+    bool moved = false;
+    if (mine) {
+        moved = ((a.pos_global[3 * t] - a.pos_local[3 * t]) |
+                 (a.pos_global[3 * t + 1] - a.pos_local[3 * t + 1]) |
+                 (a.pos_global[3 * t + 2] - a.pos_local[3 * t + 2])) != 0;
+        if (!moved && a.in_place) mine = false;
+    }
+    const int count = mine ? (l1 - lfirst + n_slots - 1) / n_slots : 0;
+    const __nv_bfloat16 *src = static_cast<const __nv_bfloat16 *>(a.k_in);
+    __nv_bfloat16 *dst = static_cast<__nv_bfloat16 *>(a.k_out);
+    const long long row0 = (static_cast<long long>(t) * a.hkv + h) * 128 + pg * 8;
+    const long long lstep = static_cast<long long>(n_slots) * a.layer_stride;
+    const long long obase = static_cast<long long>(lfirst) * a.layer_stride + row0;
+    uint4 xv = make_uint4(0, 0, 0, 0), yv = make_uint4(0, 0, 0, 0);
+    if (count > 0) {
+        xv = __ldcs(reinterpret_cast<const uint4 *>(src + obase));
+        yv = __ldcs(reinterpret_cast<const uint4 *>(src + obase + 64));
+    }
+    const bool moved_any = build_table(a, t0, TB, s_delta, tab);
+    const bool scoring = a.score_out != nullptr && slot < n_slots && t < a.T && t >= a.cand0 &&
+                         t < a.cand0 + a.n_cand && a.score_layer >= l0 && a.score_layer < l1 &&
+                         (a.score_layer - l0) % n_slots == slot;
+    if (count > 0) stream_slices(a, src, dst, obase, lstep, count, moved, moved_any, tb, pg, tab, xv, yv);
+    if (a.score_out == nullptr || __ballot_sync(0xFFFFFFFFu, scoring) == 0) return;
+    float s1 = 0.0f, s2 = 0.0f;
+    if (scoring) {
+        const long long o = static_cast<long long>(a.score_layer) * a.layer_stride + row0;
+        const uint4 cx = *reinterpret_cast<const uint4 *>(dst + o);
+        const uint4 cy = *reinterpret_cast<const uint4 *>(dst + o + 64);
+        const __nv_bfloat16 *fr = static_cast<const __nv_bfloat16 *>(a.fresh) +
+                                  static_cast<long long>(t - a.cand0) * a.fresh_stride + h * 128 + pg * 8;
+        s1 = score_block8(__ldg(reinterpret_cast<const uint4 *>(fr)), cx);
+        s2 = score_block8(__ldg(reinterpret_cast<const uint4 *>(fr + 64)), cy);
+    }
+    for (int m = 8 * a.hkv; m >= 16; m /= 2) {   // block strides >= 16: heads h and h + m/16
+        s1 = __fadd_rn(s1, __shfl_down_sync(0xFFFFFFFFu, s1, m / 2));
+        s2 = __fadd_rn(s2, __shfl_down_sync(0xFFFFFFFFu, s2, m / 2));
+    }
+    s1 = __fadd_rn(s1, s2);   // stride 8: the two halves of a head
+#pragma unroll
+    for (int m = 4; m >= 1; m /= 2) s1 = __fadd_rn(s1, __shfl_down_sync(0xFFFFFFFFu, s1, m));
+    if (scoring && h == 0 && pg == 0) a.score_out[t - a.cand0] = s1;
+}
+
 // fp32: 16 threads per 128-element row, each owning 4 frequency pairs.
 __global__ void __launch_bounds__(kThreads) rebase_f32_kernel(RebaseArgs a, int layers_per_cta) {
     __shared__ float4 tab[kMaxTokensPerCta * 64];
@@ -355,6 +408,11 @@ __global__ void __launch_bounds__(kThreads) rebase_f32_kernel(RebaseArgs a, int 
 }
 
 }  // namespace
+
+bool rebase_fuses_score(const RebaseArgs &a, cs_dtype dt) {
+    // bf16 only, and a token's row must be whole lanes of one warp (8 lanes per head)
+    return dt == CS_DTYPE_BF16 && (a.hkv == 1 || a.hkv == 2 || a.hkv == 4);
+}
 
 cudaError_t launch_rebase(const RebaseArgs &a, cs_dtype dt, cudaStream_t s) {
     if (a.T == 0 || a.n_layers == 0) return cudaSuccess;

@@ -2,9 +2,10 @@
 
 A query composes N stored chunk caches laid out as
     [text prefix P][chunk 0] ... [chunk N-1][text suffix S],   T tokens,
-and runs the four calls of the hot path in stream order:
-  1. cs_rebase_keys      all layers' keys, in place, local -> global coordinates (Eq. 3)
-  2. cs_score_deviation  candidates = tokens of chunks 1..N-1 at the score layer (Eq. 5)
+and runs the four steps of the hot path in stream order:
+  1. re-base             all layers' keys, in place, local -> global coordinates (Eq. 3)
+  2. score               candidates = tokens of chunks 1..N-1 at the score layer (Eq. 5);
+                         1 and 2 are one call, cs_rebase_and_score (one launch)
   3. cs_select_topk      k of them, written as the first k query positions
   4. cs_repair_attention the k selected rows plus the S suffix rows over the cache (Eq. 1)
 Query tensors of the repaired rows and the fresh keys of the candidates come
@@ -27,8 +28,8 @@ import dataclasses
 
 import torch
 
-from . import (cs_rebase_keys, cs_repair_attention, cs_scatter_rows, cs_score_deviation,
-               cs_select_topk)
+from . import (cs_rebase_and_score, cs_rebase_keys, cs_repair_attention, cs_scatter_rows,
+               cs_score_deviation, cs_select_topk)
 
 POLICIES = ("3axis", "scalar1d", "naive")
 
@@ -84,13 +85,14 @@ class ComposedQuery:
         s = self.shape
         if policy not in POLICIES:
             raise ValueError(f"policy must be one of {POLICIES}")
-        if policy == "3axis":
-            cs_rebase_keys(k, pos_local, pos_global, theta=s.theta, sections=s.sections, stream=stream)
-        elif policy == "scalar1d":
-            cs_rebase_keys(k, pos_local, self.scalar_targets(), theta=s.theta, sections=s.sections,
-                           stream=stream)
-        cached = k[s.score_layer, s.cand0:s.cand0 + s.n_cand]
-        cs_score_deviation(k_fresh, cached, out=self.score, stream=stream)
+        if policy == "naive":
+            cached = k[s.score_layer, s.cand0:s.cand0 + s.n_cand]
+            cs_score_deviation(k_fresh, cached, out=self.score, stream=stream)
+        else:   # re-base and score in one launch (the score reads the rows just re-based)
+            target = pos_global if policy == "3axis" else self.scalar_targets()
+            cs_rebase_and_score(k, pos_local, target, k_fresh, s.score_layer, s.cand0,
+                                score_out=self.score, theta=s.theta, sections=s.sections,
+                                stream=stream)
         cs_select_topk(self.score, s.k, s.cand0, out=self.qpos[:s.k], stream=stream)
         if fresh_kv is not None:
             k_rows, v_rows = fresh_kv

@@ -170,3 +170,26 @@ def test_scatter_rejects_bad_arguments(cslib):
     assert call(T=0, cst=0) == cslib.CS_ERR_INVALID_ARG
     assert call(n=0, rows=None, idx=None) == cslib.CS_OK
     assert call(L=0) == cslib.CS_OK
+
+
+def test_rebase_and_score_rejects_bad_arguments(cslib):
+    L = cslib.lib()
+    r = cslib._RopeCfg(1e6, (ctypes.c_int32 * 3)(16, 24, 24))
+
+    def call(**kw):
+        a = dict(k_in=FAKE, k_out=FAKE, dt=1, L=2, stride=40 * 2 * 128, T=40, H=2, D=128, pl=FAKE,
+                 pg=FAKE, sl=1, c0=8, nc=16, fr=FAKE + (1 << 24), fs=256, out=FAKE + (1 << 25))
+        a.update(kw)
+        return L.cs_rebase_and_score(a["k_in"], a["k_out"], a["dt"], a["L"], a["stride"], a["T"],
+                                     a["H"], a["D"], a["pl"], a["pg"], ctypes.byref(r), a["sl"],
+                                     a["c0"], a["nc"], a["fr"], a["fs"], a["out"], None)
+
+    assert call(sl=2) == cslib.CS_ERR_INVALID_ARG           # score layer past the last
+    assert call(sl=-1) == cslib.CS_ERR_INVALID_ARG
+    assert call(c0=30) == cslib.CS_ERR_INVALID_ARG          # candidates past T
+    assert call(nc=-1) == cslib.CS_ERR_INVALID_ARG
+    assert call(fs=100) == cslib.CS_ERR_INVALID_ARG         # fresh rows shorter than a key row
+    assert call(fr=FAKE + 8) == cslib.CS_ERR_INVALID_ARG    # misaligned fresh rows
+    assert call(out=None) == cslib.CS_ERR_INVALID_ARG
+    assert call(D=64) == cslib.CS_ERR_UNSUPPORTED
+    assert call(L=0, nc=0) == cslib.CS_OK
