@@ -20,7 +20,9 @@ Options around the four calls:
     attention, as the recompute does layer by layer (Sec. 2);
   * shallow_recompute(): the attention part of the shallow recompute, every
     candidate as a query row over the first layers (the 2 c_a |C| T term of
-    Eq. 6), run with the same attention kernel.
+    Eq. 6), run with the same attention kernel;
+  * GraphedQuery: a whole end-to-end query (input copies, the launches, output
+    copies) captured once as a CUDA graph and replayed with one launch.
 """
 from __future__ import annotations
 
@@ -112,7 +114,37 @@ class ComposedQuery:
         return cs_repair_attention(q_cand, k[:nl], v[:nl], self._cand_pos, out=out, stream=stream)
 
 
-def compose_from_host(query: ComposedQuery, host: dict, dev: dict, out_host: dict, stream=None):
+class GraphedQuery:
+    """One whole end-to-end query captured as a CUDA graph for fixed buffers: the host->device
+    copies of k, v, q and k_fresh, the three launches of the step, and the device->host copies
+    of the output and the query positions.  replay() runs all of it with one graph launch, on
+    the current contents of the host buffers.
+
+    host / dev / out_host as for compose_from_host.  The first step runs eagerly (it also
+    performs the library's one-time set-up) before the capture."""
+
+    def __init__(self, query: ComposedQuery, host: dict, dev: dict, out_host: dict,
+                 policy="3axis"):
+        self.query, self.host, self.dev, self.out_host = query, host, dev, out_host
+        self.policy = policy
+        side = torch.cuda.Stream(device=dev["k"].device)
+        side.wait_stream(torch.cuda.current_stream(dev["k"].device))
+        with torch.cuda.stream(side):
+            self.h2d, self.d2h = compose_from_host(query, host, dev, out_host, stream=side,
+                                                   policy=policy)
+        side.synchronize()
+        self.graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(self.graph, stream=side):
+            compose_from_host(query, host, dev, out_host, stream=side, policy=policy)
+
+    def replay(self):
+        """Runs the captured query on the current stream's device (asynchronously)."""
+        self.graph.replay()
+        return self.h2d, self.d2h
+
+
+def compose_from_host(query: ComposedQuery, host: dict, dev: dict, out_host: dict, stream=None,
+                      policy="3axis"):
     """End-to-end query from host memory: copies the step's inputs in, runs it, copies the result out.
 
     host / dev: dicts with k, v, q, k_fresh (pinned host tensors / device tensors of the
@@ -126,7 +158,7 @@ def compose_from_host(query: ComposedQuery, host: dict, dev: dict, out_host: dic
             dev[name].copy_(host[name], non_blocking=True)
             h2d += host[name].numel() * host[name].element_size()
         o, qpos = query.step(dev["k"], dev["v"], dev["q"], dev["k_fresh"], dev["pos_local"],
-                             dev["pos_global"], stream=st)
+                             dev["pos_global"], stream=st, policy=policy)
         out_host["o"].copy_(o, non_blocking=True)
         out_host["qpos"].copy_(qpos, non_blocking=True)
     d2h = o.numel() * o.element_size() + qpos.numel() * qpos.element_size()
