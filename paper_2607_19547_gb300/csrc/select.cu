@@ -3,7 +3,8 @@
 // One CTA of 1024 threads (the candidate scores are a few hundred KB at most and
 // stay in L2).  Scores map to order-preserving 32-bit keys.  Thread t owns the
 // contiguous candidate range [t*per, (t+1)*per); up to 16 keys per thread stay
-// in registers, larger inputs are re-read from L2 in every pass.  Three
+// in registers, larger inputs are re-read from L2 in every pass (the histogram
+// passes read them interleaved and coalesced, eight loads in flight).  Three
 // MSB-first radix passes over 11-, 11- and 10-bit digits (one shared 2048-bin
 // histogram, warp-aggregated increments) find K*, the k-th largest key, and how
 // many keys equal to K* belong to the top k (the lowest-index ones: the
@@ -103,9 +104,21 @@ select_kernel(const uint32_t *__restrict__ score, int n, int k, int idx_base, in
                 hist_add(hist, (key >> shift) & dmask, i < cnt && (key & pmask) == prefix);
             }
         } else {
-            for (int i = 0; i < per; ++i) {   // per is uniform; lanes past n are inactive
-                const uint32_t key = i < cnt ? key_at(i) : 0u;
-                hist_add(hist, (key >> shift) & dmask, i < cnt && (key & pmask) == prefix);
+            // the histogram does not care which thread counts which key: read the keys
+            // interleaved (coalesced), eight loads in flight before their increments
+            const int rounds = (n + kThreads * 8 - 1) / (kThreads * 8);   // uniform
+            for (int rr = 0; rr < rounds; ++rr) {
+                uint32_t kb[8];
+#pragma unroll
+                for (int u = 0; u < 8; ++u) {
+                    const int i = (rr * 8 + u) * kThreads + tid;
+                    kb[u] = i < n ? order_key(__ldg(score + i)) : 0u;
+                }
+#pragma unroll
+                for (int u = 0; u < 8; ++u) {
+                    const int i = (rr * 8 + u) * kThreads + tid;
+                    hist_add(hist, (kb[u] >> shift) & dmask, i < n && (kb[u] & pmask) == prefix);
+                }
             }
         }
         __syncthreads();
@@ -140,10 +153,15 @@ select_kernel(const uint32_t *__restrict__ score, int n, int k, int idx_base, in
             eq += (i < cnt && reg[i] == kstar);
         }
     } else {
-        for (int i = 0; i < cnt; ++i) {
-            const uint32_t key = key_at(i);
-            gt += key > kstar;
-            eq += key == kstar;
+        for (int c0 = 0; c0 < cnt; c0 += 8) {   // eight loads in flight
+            uint32_t kb[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) kb[u] = c0 + u < cnt ? key_at(c0 + u) : 0u;
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                gt += c0 + u < cnt && kb[u] > kstar;
+                eq += c0 + u < cnt && kb[u] == kstar;
+            }
         }
     }
     const unsigned long long mine = (static_cast<unsigned long long>(gt) << 32) | eq;
@@ -159,9 +177,16 @@ select_kernel(const uint32_t *__restrict__ score, int n, int k, int idx_base, in
                 out[pos++] = idx_base + i0 + i;
         }
     } else {
-        for (int i = 0; i < cnt; ++i) {
-            const uint32_t key = key_at(i);
-            if (key > kstar || (key == kstar && eq_seen++ < krem)) out[pos++] = idx_base + i0 + i;
+        for (int c0 = 0; c0 < cnt; c0 += 8) {
+            uint32_t kb[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) kb[u] = c0 + u < cnt ? key_at(c0 + u) : 0u;
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const uint32_t key = kb[u];
+                if (c0 + u < cnt && (key > kstar || (key == kstar && eq_seen++ < krem)))
+                    out[pos++] = idx_base + i0 + c0 + u;
+            }
         }
     }
 }
