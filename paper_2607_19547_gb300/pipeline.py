@@ -22,7 +22,9 @@ Options around the four calls:
     candidate as a query row over the first layers (the 2 c_a |C| T term of
     Eq. 6), run with the same attention kernel;
   * GraphedQuery: a whole end-to-end query (input copies, the launches, output
-    copies) captured once as a CUDA graph and replayed with one launch.
+    copies) captured once as a CUDA graph and replayed with one launch;
+  * PipelinedQuery: the same with uploads, kernels and downloads overlapped layer
+    group by layer group on three streams, also one graph.
 """
 from __future__ import annotations
 
@@ -139,6 +141,85 @@ class GraphedQuery:
 
     def replay(self):
         """Runs the captured query on the current stream's device (asynchronously)."""
+        self.graph.replay()
+        return self.h2d, self.d2h
+
+
+class PipelinedQuery:
+    """An end-to-end query from host buffers with the copies and the kernels overlapped layer
+    group by layer group, captured as one CUDA graph.
+
+    Three streams: uploads (K, V and Q of one group of layers, the fresh keys first), compute
+    (the group's re-base; for the group holding the score layer also its score and the
+    selection; then the group's attention), downloads (the group's output, and the query
+    positions at the end).  Each group's compute waits for its uploads and each download for
+    its compute, so group g+1 uploads while group g computes and group g-1 downloads.  The
+    kernels are the same calls as ComposedQuery.step on layer slices (every call takes a
+    layer count and stride), so the result is identical.  replay() runs it all with one graph
+    launch on the current contents of the host buffers."""
+
+    def __init__(self, query: ComposedQuery, host: dict, dev: dict, out_host: dict,
+                 group_layers: int = 6, policy: str = "3axis"):
+        if policy not in POLICIES:
+            raise ValueError(f"policy must be one of {POLICIES}")
+        s = query.shape
+        self.query, self.host, self.dev, self.out_host = query, host, dev, out_host
+        L = s.n_layers
+        # the first group reaches the score layer, so the selection runs as early as possible
+        first = max(group_layers, s.score_layer + 1)
+        bounds = [0] + list(range(min(first, L), L, group_layers)) + [L]
+        self.groups = [(a, b) for a, b in zip(bounds[:-1], bounds[1:]) if b > a]
+        device = dev["k"].device
+        self.s_in, self.s_c, self.s_out = (torch.cuda.Stream(device=device) for _ in range(3))
+        self.h2d = sum(host[n].numel() * host[n].element_size() for n in ("k", "v", "q", "k_fresh"))
+        self.d2h = query.out.numel() * query.out.element_size() + query.qpos.numel() * 4
+        self.s_c.wait_stream(torch.cuda.current_stream(device))
+        with torch.cuda.stream(self.s_c):
+            self._record(policy)          # eager run: one-time set-up of the library
+        self.s_c.synchronize()
+        self.graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(self.graph, stream=self.s_c):
+            self._record(policy)
+
+    def _record(self, policy):
+        q, s, host, dev, out_host = self.query, self.query.shape, self.host, self.dev, self.out_host
+        s_in, s_c, s_out = self.s_in, self.s_c, self.s_out
+        s_in.wait_stream(s_c)
+        s_out.wait_stream(s_c)
+        with torch.cuda.stream(s_in):
+            dev["k_fresh"].copy_(host["k_fresh"], non_blocking=True)
+        for a, b in self.groups:
+            with torch.cuda.stream(s_in):
+                for n in ("k", "v", "q"):
+                    dev[n][a:b].copy_(host[n][a:b], non_blocking=True)
+            s_c.wait_stream(s_in)
+            with torch.cuda.stream(s_c):
+                k = dev["k"][a:b]
+                target = dev["pos_global"] if policy == "3axis" else q.scalar_targets()
+                if a <= s.score_layer < b:
+                    if policy == "naive":
+                        cached = dev["k"][s.score_layer, s.cand0:s.cand0 + s.n_cand]
+                        cs_score_deviation(dev["k_fresh"], cached, out=q.score, stream=s_c)
+                    else:
+                        cs_rebase_and_score(k, dev["pos_local"], target, dev["k_fresh"],
+                                            s.score_layer - a, s.cand0, score_out=q.score,
+                                            theta=s.theta, sections=s.sections, stream=s_c)
+                    cs_select_topk(q.score, s.k, s.cand0, out=q.qpos[:s.k], stream=s_c)
+                elif policy != "naive":
+                    cs_rebase_keys(k, dev["pos_local"], target, theta=s.theta, sections=s.sections,
+                                   stream=s_c)
+                cs_repair_attention(dev["q"][a:b], k, dev["v"][a:b], q.qpos, out=q.out[a:b],
+                                    stream=s_c)
+            s_out.wait_stream(s_c)
+            with torch.cuda.stream(s_out):
+                out_host["o"][a:b].copy_(q.out[a:b], non_blocking=True)
+        with torch.cuda.stream(s_out):
+            out_host["qpos"].copy_(q.qpos, non_blocking=True)
+        s_c.wait_stream(s_in)
+        s_c.wait_stream(s_out)
+
+    def replay(self):
+        """Runs the captured query (asynchronously, ordered after the current stream's work)."""
         self.graph.replay()
         return self.h2d, self.d2h
 

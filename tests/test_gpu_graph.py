@@ -69,3 +69,33 @@ def test_graph_replay_equals_eager(cslib, name):
         assert np.array_equal(bits16(got["o"]), bits16(eager["o"]))
     else:
         assert torch.equal(got["o"], eager["o"])
+
+
+@pytest.mark.parametrize("name,policy,group", [("tiny_f32", "3axis", 6), ("qwen3b_4x1024", "3axis", 6),
+                                               ("qwen3b_4x1024", "scalar1d", 5),
+                                               ("qwen3b_4x1024", "naive", 36)])
+def test_pipelined_query_equals_eager(cslib, name, policy, group):
+    """Uploads, kernels and downloads overlapped layer group by layer group (one graph) give the
+    eager query's result bit for bit."""
+    from paper_2607_19547_gb300.pipeline import PipelinedQuery
+    w = W.CONFIGS[name]
+    shape, host, dev = _setup(w, 31)
+    qe = ComposedQuery(shape, w.torch_dtype)
+    eager = _out_host(qe, w)
+    dev_e = {k: (v.clone() if k in ("k", "v", "q", "k_fresh") else v) for k, v in dev.items()}
+    compose_from_host(qe, host, dev_e, eager, policy=policy)
+    torch.cuda.synchronize()
+    qp = ComposedQuery(shape, w.torch_dtype)
+    got = _out_host(qp, w)
+    pq = PipelinedQuery(qp, host, dev, got, group_layers=group, policy=policy)
+    for _ in range(2):
+        for t in got.values():
+            t.zero_()
+        pq.replay()
+        torch.cuda.synchronize()
+        cslib.cs_sync_status()
+        assert np.array_equal(got["qpos"].numpy(), eager["qpos"].numpy())
+        if w.dtype == "bf16":
+            assert np.array_equal(bits16(got["o"]), bits16(eager["o"]))
+        else:
+            assert torch.equal(got["o"], eager["o"])
