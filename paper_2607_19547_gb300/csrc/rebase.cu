@@ -79,35 +79,61 @@ __device__ void sincos_turns(unsigned long long u, f2 &sn, f2 &cs) {
 // bf16 bits of u*c - w*s from the double-float evaluation (c = c_hi + c_lo,
 // s = s_hi + s_lo), rounded once: the error-free products and sum carry the
 // value to about 2^-44 relative, far inside any rounding decision left to it.
+// When the leading sum already overflows fp32 (|p - q| >= 2^128 - 2^103), the
+// exact value lies beyond the bf16 overflow threshold 2^128 - 2^119 as well,
+// so the result is that infinity (the error terms would turn into NaN).
 __device__ __forceinline__ uint32_t rot_bf16_df(float u, float w, float4 cs4) {
     const f2 p = two_prod(u, cs4.x);
     const f2 q = two_prod(w, cs4.z);
     const f2 d = two_sum(p.hi, -q.hi);
+    if (isinf(d.hi)) return __float_as_uint(d.hi) >> 16;
     const float tail = __fadd_rn(__fadd_rn(__fsub_rn(p.lo, q.lo), d.lo),
                                  __fsub_rn(__fmul_rn(u, cs4.y), __fmul_rn(w, cs4.w)));
     const f2 rr = two_sum(d.hi, tail);
     return bf16_round_f2(rr.hi, rr.lo);
 }
 
-struct Row8 {
-    uint32_t w[8];   // 4 words of first-half outputs, then 4 of second-half outputs
-};
+// Slices whose bf16 rounding was uncertain wait in a per-warp queue in shared
+// memory (their raw input words and where they came from) and are redone by the
+// whole warp together, one output pair per lane, so the rare slow path never runs
+// on one lane while the other 31 wait.
+constexpr int kQueue = 64;   // entries per warp
 
-// One thread's slice (8 pairs) rotated entirely in double-float and rounded
-// once; kept out of line because only a few slices in ten thousand need it.
-__device__ __noinline__ Row8 rot_row_df(uint4 xv, uint4 yv, const float4 *full) {
-    const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w};
-    const uint32_t yw[4] = {yv.x, yv.y, yv.z, yv.w};
-    Row8 out;
-#pragma unroll
-    for (int w = 0; w < 4; ++w) {
-        const float xa = bf16_lo(xw[w]), xb = bf16_hi(xw[w]);
-        const float ya = bf16_lo(yw[w]), yb = bf16_hi(yw[w]);
-        const float4 ca = full[2 * w], cb = full[2 * w + 1];
-        out.w[w] = rot_bf16_df(xa, ya, ca) | (rot_bf16_df(xb, yb, cb) << 16);
-        out.w[4 + w] = rot_bf16_df(ya, -xa, ca) | (rot_bf16_df(yb, -xb, cb) << 16);
+__shared__ uint4 q_xy[kThreads / 32][2 * kQueue];   // first- and second-half words
+__shared__ uint32_t q_meta[kThreads / 32][kQueue];  // (slice index << 5) | owning lane
+
+// Rotates the n queued slices of this warp entirely in double-float, rounds each
+// output once and stores it.  Called by exactly the lanes of `part` (the lanes
+// that rotate), each passing its own output offset `obase` and table row `trow`.
+__device__ __forceinline__ void redo_queue(int n, unsigned part, long long obase,
+                                        long long lstep, int trow, const float4 *tab,
+                                        __nv_bfloat16 *dst) {
+    __syncwarp(part);   // entries written by other lanes
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int rank = __popc(part & ((1u << lane) - 1u));
+    const int nl = __popc(part);
+    const int items = n * 8;   // 8 frequency pairs per slice
+    uint16_t *d16 = reinterpret_cast<uint16_t *>(dst);
+    for (int base = 0; base < items; base += nl) {   // the same trip count on every lane
+        const int it = base + rank;
+        const bool valid = it < items;
+        const int ent = valid ? it >> 3 : 0, p = it & 7;
+        const uint32_t mt = q_meta[warp][ent];
+        const int olane = static_cast<int>(mt & 31u);
+        const long long ob = __shfl_sync(part, obase, olane);
+        const int orow = __shfl_sync(part, trow, olane);
+        if (valid) {
+            const uint32_t *w = reinterpret_cast<const uint32_t *>(&q_xy[warp][2 * ent]);
+            const uint32_t xw = w[p >> 1], yw = w[4 + (p >> 1)];
+            const float x = (p & 1) ? bf16_hi(xw) : bf16_lo(xw);
+            const float y = (p & 1) ? bf16_hi(yw) : bf16_lo(yw);
+            const float4 cs4 = tab[orow + p];
+            const long long o = ob + static_cast<long long>(mt >> 5) * lstep + p;
+            d16[o] = static_cast<uint16_t>(rot_bf16_df(x, y, cs4));
+            d16[o + 64] = static_cast<uint16_t>(rot_bf16_df(y, -x, cs4));
+        }
     }
-    return out;
+    __syncwarp(part);   // the queue is reused; later reads of these rows see the stores
 }
 
 // Two fp32 values rounded to nearest-even bf16 and packed (lo in bits 0-15).
@@ -117,11 +143,13 @@ __device__ __forceinline__ uint32_t pack_bf16x2_rn(float lo, float hi) {
     return r;
 }
 
-// fp32 result of u*c - w*s from the double-float evaluation.
+// fp32 result of u*c - w*s from the double-float evaluation (an overflowing
+// leading sum is returned as the infinity it rounds to, as above).
 __device__ __forceinline__ float rot_f32(float u, float w, float4 cs4) {
     const f2 p = two_prod(u, cs4.x);
     const f2 q = two_prod(w, cs4.z);
     const f2 d = two_sum(p.hi, -q.hi);
+    if (isinf(d.hi)) return d.hi;
     const float tail = __fadd_rn(__fadd_rn(__fsub_rn(p.lo, q.lo), d.lo),
                                  __fsub_rn(__fmul_rn(u, cs4.y), __fmul_rn(w, cs4.w)));
     return __fadd_rn(d.hi, tail);
@@ -173,20 +201,29 @@ __device__ bool build_table(const RebaseArgs &a, int t0, int TB, int (*s_delta)[
 // half: elements i) and yv (second half: elements i + 64).  Returns false if
 // the bf16 rounding of any output is uncertain.
 //
-// Each output r ~ u c - w s is evaluated in fp32 with |error| <= E, where
-// E = (|x| + |y|) * 2.5 * 2^-24 (product and fma roundings plus
-// |c - c_hi|, |s - s_hi| <= 2^-25), bounded here by (|x| + |y|) * 2^-22.  The
-// bf16 rounding is certain when no bf16 midpoint lies within E of r: the
-// midpoint of r's interval is (|r| truncated to bf16) + half a bf16 unit, an
-// fp32 number in r's binade, so |r| - mid is exact; requiring |r| > 2048 E
-// keeps the neighbouring intervals' midpoints (at least |r| / 1024 away) out
-// of reach too.  A NaN or infinite r fails.
+// Each output r ~ u c - w s is evaluated in fp32 with
+//   |r - exact| <= 2.5 * 2^-24 * (|x| + |y|) + 2^-149
+// (c_hi and s_hi lie within 2^-25 of cos and sin; one rounding of the product,
+// one of the fma; the last term covers subnormal results), so
+// E = 3 * 2^-24 * fl(|x| + |y|) + 2^-148, rounded once, exceeds the error
+// strictly.  The bf16 rounding of r is certain when
+//   (1) the midpoint m of r's own bf16 interval (|r| truncated to bf16 plus half
+//       a bf16 unit: an fp32 number in r's binade, so |r| - m is exact) lies at
+//       least E away from |r|, and
+//   (2) |r| >= 1024 E: for |r| in [2^e, 2^(e+1)) this makes E < 2^(e-9), the
+//       least distance from r to any other midpoint (the one just below a power
+//       of two included; subnormal r alike, with midpoints 2^-134 apart).
+// Each condition is a difference that rounds to a negative number exactly when
+// it fails, so the sign bits of all 32 differences are OR-ed and tested once.
+// Non-finite and huge inputs (where r could overflow) fail through the sum of
+// |x| + |y| over the slice, which must compare below 2^126 (NaN compares false).
 __device__ __forceinline__ bool rotate_slice(const uint4 &xv, const uint4 &yv, const float (&c)[8],
                                              const float (&sn)[8], uint32_t (&ow)[4],
                                              uint32_t (&pw)[4]) {
     const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w};
     const uint32_t yw[4] = {yv.x, yv.y, yv.z, yv.w};
-    bool ok = true;
+    uint32_t neg = 0;
+    float usum = 0.0f;
 #pragma unroll
     for (int w = 0; w < 4; ++w) {
         float r1[2], r2[2];
@@ -197,17 +234,22 @@ __device__ __forceinline__ bool rotate_slice(const uint4 &xv, const uint4 &yv, c
             const float y = h ? bf16_hi(yw[w]) : bf16_lo(yw[w]);
             r1[h] = __fmaf_rn(x, c[e], -__fmul_rn(y, sn[e]));    // x c - y s
             r2[h] = __fmaf_rn(y, c[e], __fmul_rn(x, sn[e]));     // y c + x s
-            const float E = __fmul_rn(__fadd_rn(fabsf(x), fabsf(y)), 0x1p-22f);
-            const float E2 = __fmul_rn(E, 2048.0f);
+            const float u = __fadd_rn(fabsf(x), fabsf(y));
+            usum = __fadd_rn(usum, u);
+            const float E = __fmaf_rn(u, 0x1.8p-23f, 0x1p-148f);
+            const float E2 = __fmul_rn(E, 1024.0f);
+            const float a1 = fabsf(r1[h]), a2 = fabsf(r2[h]);
             const float m1 = __uint_as_float((__float_as_uint(r1[h]) & 0x7FFF0000u) | 0x8000u);
             const float m2 = __uint_as_float((__float_as_uint(r2[h]) & 0x7FFF0000u) | 0x8000u);
-            ok = ok & (fabsf(__fsub_rn(fabsf(r1[h]), m1)) > E) & (fabsf(r1[h]) > E2) &
-                 (fabsf(__fsub_rn(fabsf(r2[h]), m2)) > E) & (fabsf(r2[h]) > E2);
+            neg |= __float_as_uint(__fsub_rn(fabsf(__fsub_rn(a1, m1)), E)) |
+                   __float_as_uint(__fsub_rn(a1, E2));
+            neg |= __float_as_uint(__fsub_rn(fabsf(__fsub_rn(a2, m2)), E)) |
+                   __float_as_uint(__fsub_rn(a2, E2));
         }
         ow[w] = pack_bf16x2_rn(r1[0], r1[1]);
         pw[w] = pack_bf16x2_rn(r2[0], r2[1]);
     }
-    return ok;
+    return (neg >> 31) == 0 && usum < 0x1p126f;
 }
 
 // Eq. 5 block term of the canonical fp32 order: ((q0+q1)+(q2+q3))+((q4+q5)+(q6+q7)),
@@ -227,10 +269,12 @@ __device__ __forceinline__ float score_block8(uint4 fv, uint4 cv) {
                      __fadd_rn(__fadd_rn(q[4], q[5]), __fadd_rn(q[6], q[7])));
 }
 
-// The streaming part of the bf16 kernel for one thread's slices (see the kernel below).
-__device__ __forceinline__ void stream_slices(const RebaseArgs &a, const __nv_bfloat16 *src,
-                                              __nv_bfloat16 *dst, long long obase, long long lstep,
-                                              int count, bool moved, bool moved_any, int tb, int pg,
+// The streaming part of the bf16 kernel for one thread's slices (see the kernel
+// below).  `part` holds the lanes of this warp that rotate (moved tokens with
+// layers to walk); they all walk the same number of layers.
+__device__ __forceinline__ void stream_slices(const __nv_bfloat16 *src, __nv_bfloat16 *dst,
+                                              long long obase, long long lstep, int count,
+                                              bool moved, unsigned part, int trow,
                                               const float4 *tab, uint4 xv, uint4 yv) {
     if (!moved) {   // out-of-place copy of an unmoved token
         for (int i = 0; i < count; ++i) {
@@ -244,42 +288,46 @@ __device__ __forceinline__ void stream_slices(const RebaseArgs &a, const __nv_bf
         }
         return;
     }
-    (void)moved_any;   // a moved token implies the table was built
-    const float4 *full = &tab[tb * 64 + pg * 8];
+    const float4 *full = &tab[trow];
     float c[8], sn[8];
 #pragma unroll
     for (int e = 0; e < 8; ++e) {
         c[e] = full[e].x;
         sn[e] = full[e].z;
     }
-    unsigned long long redo = 0;   // the host keeps count <= 64
+    int queued = 0;   // the same on every lane of `part`
     for (int i = 0; i < count; ++i) {
+        if (queued > kQueue - 32) {   // make room for one failing slice per lane
+            redo_queue(queued, part, obase, lstep, trow, tab, dst);
+            queued = 0;
+        }
         uint4 xn = make_uint4(0, 0, 0, 0), yn = make_uint4(0, 0, 0, 0);
         if (i + 1 < count) {
             xn = __ldcs(reinterpret_cast<const uint4 *>(src + obase + (i + 1) * lstep));
             yn = __ldcs(reinterpret_cast<const uint4 *>(src + obase + (i + 1) * lstep + 64));
         }
         uint32_t ow[4], pw[4];
-        if (rotate_slice(xv, yv, c, sn, ow, pw)) {
+        const bool ok = rotate_slice(xv, yv, c, sn, ow, pw);
+        if (ok) {
             const long long o = obase + i * lstep;
             __stcs(reinterpret_cast<uint4 *>(dst + o), make_uint4(ow[0], ow[1], ow[2], ow[3]));
             __stcs(reinterpret_cast<uint4 *>(dst + o + 64), make_uint4(pw[0], pw[1], pw[2], pw[3]));
-        } else {
-            redo |= 1ull << i;
+        }
+        const unsigned fails = __ballot_sync(part, !ok);
+        if (fails) {   // rare: queue the uncertain slices (not stored) for the warp to redo
+            if (!ok) {
+                const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+                const int e = queued + __popc(fails & ((1u << lane) - 1u));
+                q_xy[warp][2 * e] = xv;
+                q_xy[warp][2 * e + 1] = yv;
+                q_meta[warp][e] = (static_cast<uint32_t>(i) << 5) | static_cast<uint32_t>(lane);
+            }
+            queued += __popc(fails);
         }
         xv = xn;
         yv = yn;
     }
-    while (redo) {   // rare: slices whose rounding was uncertain, redone in double-float
-        const int i = __ffsll(static_cast<long long>(redo)) - 1;
-        redo &= redo - 1;
-        const long long o = obase + i * lstep;
-        const uint4 x0 = *reinterpret_cast<const uint4 *>(src + o);
-        const uint4 y0 = *reinterpret_cast<const uint4 *>(src + o + 64);
-        const Row8 rr = rot_row_df(x0, y0, full);
-        *reinterpret_cast<uint4 *>(dst + o) = make_uint4(rr.w[0], rr.w[1], rr.w[2], rr.w[3]);
-        *reinterpret_cast<uint4 *>(dst + o + 64) = make_uint4(rr.w[4], rr.w[5], rr.w[6], rr.w[7]);
-    }
+    if (queued) redo_queue(queued, part, obase, lstep, trow, tab, dst);
 }
 
 // bf16: 8 threads per 128-element row, each owning 8 frequency pairs (16 bytes
@@ -290,9 +338,9 @@ __device__ __forceinline__ void stream_slices(const RebaseArgs &a, const __nv_bf
 //   - each thread reads its own token's delta and issues its first load before
 //     the table is built, so DRAM latency overlaps the sincos evaluation;
 //   - the next layer's slice is loaded before the current one is rotated;
-//   - a slice with an uncertain rounding is not stored; its layer is recorded
-//     and, after the streaming loop, redone in double-float from the untouched
-//     input (keeping the rare slow path out of the hot loop);
+//   - a slice with an uncertain rounding is not stored; its input words go to
+//     the warp's redo queue and the whole warp redoes the queued slices in
+//     double-float when the queue fills and after the streaming loop;
 //   - with the fused score, the slot that re-based layer score_layer reads its
 //     candidate rows back (its own stores) with the matching fresh rows and
 //     reduces each token's 16 * n_kv_heads block sums in the canonical halving
@@ -338,7 +386,10 @@ __global__ void __launch_bounds__(kThreads, 4) rebase_bf16_kernel(RebaseArgs a, 
     const bool scoring = a.score_out != nullptr && slot < n_slots && t < a.T && t >= a.cand0 &&
                          t < a.cand0 + a.n_cand && a.score_layer >= l0 && a.score_layer < l1 &&
                          (a.score_layer - l0) % n_slots == slot;
-    if (count > 0) stream_slices(a, src, dst, obase, lstep, count, moved, moved_any, tb, pg, tab, xv, yv);
+    // build_table ended with a block barrier: every lane takes part in this ballot
+    const unsigned part = __ballot_sync(0xFFFFFFFFu, count > 0 && moved && moved_any);
+    if (count > 0)
+        stream_slices(src, dst, obase, lstep, count, moved, part, tb * 64 + pg * 8, tab, xv, yv);
     if (a.score_out == nullptr || __ballot_sync(0xFFFFFFFFu, scoring) == 0) return;
     float s1 = 0.0f, s2 = 0.0f;
     if (scoring) {
@@ -427,8 +478,6 @@ cudaError_t launch_rebase(const RebaseArgs &a, cs_dtype dt, cudaStream_t s) {
         const int target = 152 * 2;
         if (blocks < target) groups = std::min((target + blocks - 1) / blocks,
                                                (a.n_layers + slots - 1) / slots);
-        // each thread walks at most 64 layers (its redo mask is 64 bits)
-        groups = std::max(groups, (a.n_layers + 64 * slots - 1) / (64 * slots));
         const int l_per_cta = (a.n_layers + groups - 1) / groups;
         dim3 grid(blocks, (a.n_layers + l_per_cta - 1) / l_per_cta);
         rebase_bf16_kernel<<<grid, kThreads, 0, s>>>(a, TB, l_per_cta);

@@ -133,3 +133,80 @@ def test_large_configs_sampled_tokens(cslib, name):
     exp_r, exp_x = O.rebase(before, loc[tokens], glo[tokens], "bf16")
     assert np.max(np.abs(f64(got) - exp_x)) <= TOL["bf16"]
     assert int(np.sum(bits16(got) != O.bf16_bits(exp_r))) == 0
+
+
+def _hard_pairs(L, T, H, loc, glo, seed):
+    """bf16 keys [L, T, H, 128] whose rotations often land where the fp32 fast path cannot
+    decide the bf16 rounding: exact zeros, subnormal and tiny values, values near the top of
+    the bf16 range, and pairs chosen so that one output of the rotation nearly cancels."""
+    rng = np.random.default_rng(seed)
+    shape = (L, T, H, 64)
+    x = rng.standard_normal(shape)
+    y = rng.standard_normal(shape)
+    cls = rng.integers(0, 8, size=shape)
+
+    def mag(lo, hi):
+        return np.exp2(rng.uniform(lo, hi, size=shape)) * rng.choice([-1.0, 1.0], size=shape)
+
+    theta = O.rope_theta(1e6, 128)
+    ang = (glo - loc).astype(np.float64)[:, O.axis_of_pair((16, 24, 24))] * theta   # [T, 64]
+    c, s = np.cos(ang)[None, :, None, :], np.sin(ang)[None, :, None, :]
+    with np.errstate(divide="ignore", invalid="ignore"):
+        cancel1 = np.clip(np.where(np.abs(s) > 1e-6, x * c / s, 0.0), -1e30, 1e30)    # x c - y s ~ 0
+        cancel2 = np.clip(np.where(np.abs(s) > 1e-6, -y * c / s, 0.0), -1e30, 1e30)   # y c + x s ~ 0
+    x = np.where(cls == 0, 0.0, x)
+    y = np.where(cls == 0, 0.0, y)
+    y = np.where(cls == 1, 0.0, y)
+    x = np.where(cls == 2, mag(-133, -126), x)
+    y = np.where(cls == 2, mag(-133, -118), y)
+    x = np.where(cls == 3, mag(100, 127.9), x)
+    y = np.where(cls == 3, mag(100, 127.9), y)
+    y = np.where(cls == 4, cancel1, y)
+    x = np.where(cls == 5, cancel2, x)
+    k = np.concatenate([x, y], axis=-1)
+    return torch.tensor(k, dtype=torch.float64).to(torch.float32).to(torch.bfloat16)
+
+
+@pytest.mark.parametrize("H", [1, 2, 4])
+@pytest.mark.parametrize("out_of_place", [False, True])
+def test_rounding_hard_cases_bit_exact(cslib, H, out_of_place):
+    """Most slices here fail the fp32 rounding test, so the per-warp redo queue fills and is
+    drained inside the layer loop many times; every output must still be the correctly
+    rounded rotation, bit for bit (the max-abs bound does not apply to keys near 2^127)."""
+    L, T = 16, 101
+    loc, glo = W.random_coordinates(T, seed=40 + H, max_coord=3000)
+    glo[::9] = loc[::9]
+    k = _hard_pairs(L, T, H, loc, glo, seed=H).cuda()
+    before = f64(k)
+    assert np.all(np.isfinite(before))
+    if out_of_place:
+        res = cslib.cs_rebase_keys(k, cuda(loc), cuda(glo), k_out=torch.empty_like(k))
+    else:
+        res = cslib.cs_rebase_keys(k, cuda(loc), cuda(glo))
+    cslib.cs_sync_status()
+    exp_r, _ = O.rebase(before, loc, glo, "bf16")
+    # an exactly zero rotation may come out as +0 or -0: compare zeros by value
+    gb = np.where(bits16(res) == 0x8000, 0, bits16(res))
+    eb = np.where(O.bf16_bits(exp_r) == 0x8000, 0, O.bf16_bits(exp_r))
+    bad = gb != eb
+    assert int(np.sum(bad)) == 0, (int(np.sum(bad)), gb[bad][:8], eb[bad][:8],
+                                   before[..., :64][bad[..., :64]][:8],
+                                   before[..., 64:][bad[..., :64]][:8])
+
+
+def test_rounding_hard_cases_f32(cslib):
+    """fp32 storage on the same hard inputs: within 2^-22 relative (plus an absolute 2^-140
+    for subnormal results) of the exact rotation, and the infinity where it overflows."""
+    L, T, H = 6, 77, 2
+    loc, glo = W.random_coordinates(T, seed=77, max_coord=3000)
+    k = _hard_pairs(L, T, H, loc, glo, seed=9).to(torch.float32).cuda()
+    before = f64(k)
+    res = cslib.cs_rebase_keys(k, cuda(loc), cuda(glo))
+    cslib.cs_sync_status()
+    exact = O.rebase_f64(before, loc, glo)
+    expect = np.where(np.abs(exact) >= 2.0 ** 128 - 2.0 ** 103, np.copysign(np.inf, exact), exact)
+    got = f64(res)
+    inf = np.isinf(expect)
+    assert np.array_equal(got[inf], expect[inf])
+    err = np.abs(got[~inf] - expect[~inf])
+    assert np.all(err <= np.abs(expect[~inf]) * 2.0 ** -22 + 2.0 ** -140)
