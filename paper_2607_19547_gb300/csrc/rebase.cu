@@ -296,6 +296,7 @@ __device__ __forceinline__ void stream_slices(const __nv_bfloat16 *src, __nv_bfl
         sn[e] = full[e].z;
     }
     int queued = 0;   // the same on every lane of `part`
+#pragma unroll 2
     for (int i = 0; i < count; ++i) {
         if (queued > kQueue - 32) {   // make room for one failing slice per lane
             redo_queue(queued, part, obase, lstep, trow, tab, dst);
