@@ -82,6 +82,18 @@ def test_random_coordinates_ragged(cslib, H, dtype):
     _check(cslib, k.clone(), loc, glo, name, layer_pad=5)
 
 
+@pytest.mark.parametrize("H", [8, 16, 32])
+def test_many_kv_heads_bf16(cslib, H):
+    """Up to the 32 kv heads the bf16 kernel accepts: one token per block, 1-4 layer slots."""
+    T, L = 37, 5
+    g = torch.Generator(device="cuda").manual_seed(500 + H)
+    k = torch.randn((L, T, H, 128), generator=g, device="cuda").to(torch.bfloat16)
+    loc, glo = W.random_coordinates(T, seed=H, max_coord=4000)
+    glo[::5] = loc[::5]
+    _check(cslib, k.clone(), loc, glo, "bf16")
+    _check(cslib, k.clone(), loc, glo, "bf16", out_of_place=True)
+
+
 def test_extreme_deltas(cslib):
     T = 64
     k = torch.randn((2, T, 2, 128), device="cuda").to(torch.bfloat16)

@@ -17,7 +17,7 @@ def _rows(n, H, dtype, seed, scale=1.0):
     return (torch.randn((n, H, 128), generator=g, device="cuda") * scale).to(dtype)
 
 
-@pytest.mark.parametrize("H", [1, 2, 4, 7, 8])
+@pytest.mark.parametrize("H", [1, 2, 4, 7, 8, 16])
 @pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
 @pytest.mark.parametrize("n", [1, 37, 3072])
 def test_score_bit_exact(cslib, H, dtype, n):
