@@ -24,7 +24,7 @@ Options around the four calls:
   * GraphedQuery: a whole end-to-end query (input copies, the launches, output
     copies) captured once as a CUDA graph and replayed with one launch;
   * PipelinedQuery: the same with uploads, kernels and downloads overlapped layer
-    group by layer group on three streams, also one graph.
+    group by layer group on three streams (short first and last groups), also one graph.
 """
 from __future__ import annotations
 
@@ -159,16 +159,30 @@ class PipelinedQuery:
     launch on the current contents of the host buffers."""
 
     def __init__(self, query: ComposedQuery, host: dict, dev: dict, out_host: dict,
-                 group_layers: int = 6, policy: str = "3axis"):
+                 group_layers: int = 4, policy: str = "3axis", bounds=None):
         if policy not in POLICIES:
             raise ValueError(f"policy must be one of {POLICIES}")
         s = query.shape
         self.query, self.host, self.dev, self.out_host = query, host, dev, out_host
         L = s.n_layers
-        # the first group reaches the score layer, so the selection runs as early as possible
-        first = max(group_layers, s.score_layer + 1)
-        bounds = [0] + list(range(min(first, L), L, group_layers)) + [L]
-        self.groups = [(a, b) for a, b in zip(bounds[:-1], bounds[1:]) if b > a]
+        if bounds is None:
+            # a short first group that reaches the score layer (the pipeline waits for its
+            # upload; the selection runs as early as possible), groups of group_layers, and
+            # a short last group (its compute and download trail the last upload)
+            lead, tail = min(L, max(2, s.score_layer + 1)), 2
+            bounds = [0, lead]
+            while bounds[-1] + group_layers < L - tail:
+                bounds.append(bounds[-1] + group_layers)
+            if L - tail > bounds[-1]:
+                bounds.append(L - tail)
+            if L > bounds[-1]:
+                bounds.append(L)
+        bounds = list(bounds)
+        if bounds[0] != 0 or bounds[-1] != L or any(b <= a for a, b in zip(bounds[:-1], bounds[1:])):
+            raise ValueError("bounds must rise strictly from 0 to n_layers")
+        if not any(a <= s.score_layer < b for a, b in zip(bounds[:-1], bounds[1:])):
+            raise ValueError("the score layer must lie in a group")
+        self.groups = list(zip(bounds[:-1], bounds[1:]))
         device = dev["k"].device
         self.s_in, self.s_c, self.s_out = (torch.cuda.Stream(device=device) for _ in range(3))
         self.h2d = sum(host[n].numel() * host[n].element_size() for n in ("k", "v", "q", "k_fresh"))
