@@ -349,18 +349,24 @@ __device__ __forceinline__ void stream_slices(const __nv_bfloat16 *src, __nv_bfl
 //     strides of 16 and more blocks are lane offsets of 8 and 16, the stride of
 //     8 blocks stays inside a thread (its two halves), and 4, 2, 1 are lane
 //     offsets again.
-__global__ void __launch_bounds__(kThreads, 4) rebase_bf16_kernel(RebaseArgs a, int TB, int l_per_cta) {
+// HKV > 0: the kv head count is that compile-time constant (the token block is
+// then 8 / HKV tokens, 64 threads per layer slot, and the index arithmetic below
+// is shifts); HKV == 0: any head count, TB as passed.
+template <int HKV>
+__global__ void __launch_bounds__(kThreads, 4) rebase_bf16_kernel(RebaseArgs a, int TB_arg, int l_per_cta) {
+    const int hkv = HKV > 0 ? HKV : a.hkv;
+    const int TB = HKV > 0 ? 8 / HKV : TB_arg;
     __shared__ float4 tab[kMaxTokensBf16 * 64];
     __shared__ int s_delta[kMaxTokensBf16][3];
     const int t0 = blockIdx.x * TB;
     const int l0 = blockIdx.y * l_per_cta;
     const int l1 = min(a.n_layers, l0 + l_per_cta);
-    const int slot_threads = TB * a.hkv * 8;
+    const int slot_threads = TB * hkv * 8;
     const int n_slots = kThreads / slot_threads;
     const int slot = threadIdx.x / slot_threads;
     const int loc = threadIdx.x - slot * slot_threads;
-    const int tb = loc / (a.hkv * 8);
-    const int h = (loc >> 3) % a.hkv;
+    const int tb = loc / (hkv * 8);
+    const int h = (loc >> 3) % hkv;
     const int pg = loc & 7;
     const int t = t0 + tb;
     const int lfirst = l0 + slot;
@@ -375,7 +381,7 @@ __global__ void __launch_bounds__(kThreads, 4) rebase_bf16_kernel(RebaseArgs a, 
     const int count = mine ? (l1 - lfirst + n_slots - 1) / n_slots : 0;
     const __nv_bfloat16 *src = static_cast<const __nv_bfloat16 *>(a.k_in);
     __nv_bfloat16 *dst = static_cast<__nv_bfloat16 *>(a.k_out);
-    const long long row0 = (static_cast<long long>(t) * a.hkv + h) * 128 + pg * 8;
+    const long long row0 = (static_cast<long long>(t) * hkv + h) * 128 + pg * 8;
     const long long lstep = static_cast<long long>(n_slots) * a.layer_stride;
     const long long obase = static_cast<long long>(lfirst) * a.layer_stride + row0;
     uint4 xv = make_uint4(0, 0, 0, 0), yv = make_uint4(0, 0, 0, 0);
@@ -402,7 +408,7 @@ __global__ void __launch_bounds__(kThreads, 4) rebase_bf16_kernel(RebaseArgs a, 
         s1 = score_block8(__ldg(reinterpret_cast<const uint4 *>(fr)), cx);
         s2 = score_block8(__ldg(reinterpret_cast<const uint4 *>(fr + 64)), cy);
     }
-    for (int m = 8 * a.hkv; m >= 16; m /= 2) {   // block strides >= 16: heads h and h + m/16
+    for (int m = 8 * hkv; m >= 16; m /= 2) {   // block strides >= 16: heads h and h + m/16
         s1 = __fadd_rn(s1, __shfl_down_sync(0xFFFFFFFFu, s1, m / 2));
         s2 = __fadd_rn(s2, __shfl_down_sync(0xFFFFFFFFu, s2, m / 2));
     }
@@ -481,7 +487,12 @@ cudaError_t launch_rebase(const RebaseArgs &a, cs_dtype dt, cudaStream_t s) {
                                                (a.n_layers + slots - 1) / slots);
         const int l_per_cta = (a.n_layers + groups - 1) / groups;
         dim3 grid(blocks, (a.n_layers + l_per_cta - 1) / l_per_cta);
-        rebase_bf16_kernel<<<grid, kThreads, 0, s>>>(a, TB, l_per_cta);
+        switch (a.hkv) {
+            case 1: rebase_bf16_kernel<1><<<grid, kThreads, 0, s>>>(a, TB, l_per_cta); break;
+            case 2: rebase_bf16_kernel<2><<<grid, kThreads, 0, s>>>(a, TB, l_per_cta); break;
+            case 4: rebase_bf16_kernel<4><<<grid, kThreads, 0, s>>>(a, TB, l_per_cta); break;
+            default: rebase_bf16_kernel<0><<<grid, kThreads, 0, s>>>(a, TB, l_per_cta); break;
+        }
     } else {
         const int TB = a.hkv >= kMaxTokensPerCta / 2 ? 1 : (kMaxTokensPerCta / 2) / a.hkv;
         const int layers_per_cta = 4;
