@@ -6,7 +6,7 @@
 // in registers, larger inputs are re-read from L2 in every pass (the histogram
 // passes read them interleaved and coalesced, eight loads in flight).  Three
 // MSB-first radix passes over 11-, 11- and 10-bit digits (one shared 2048-bin
-// histogram, warp-aggregated increments) find K*, the k-th largest key, and how
+// histogram, shared-memory atomic increments) find K*, the k-th largest key, and how
 // many keys equal to K* belong to the top k (the lowest-index ones: the
 // tie-break).  One block-wide scan of the per-thread (greater, equal) counts
 // then gives every selected index its output position, so the output is
@@ -28,13 +28,12 @@ __device__ __forceinline__ uint32_t order_key(uint32_t u) {
     return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
-// hist[d] += 1 for every lane with `active`; lanes sharing a digit add once.
+// hist[d] += 1 for every lane with `active`.  Plain shared-memory atomics: lanes
+// that share a digit (scores of one binade often do) were measured faster this way
+// than aggregated with __match_any_sync first (10.7 / 18.3 / 59.7 us against 12.6 /
+// 29.0 / 112 us for 3 072 / 15 360 / 64 512 candidates).
 __device__ __forceinline__ void hist_add(uint32_t *hist, uint32_t d, bool active) {
-    const uint32_t am = __ballot_sync(0xFFFFFFFFu, active);
-    if (active) {
-        const uint32_t peers = __match_any_sync(am, d);
-        if ((threadIdx.x & 31) == __ffs(peers) - 1) atomicAdd(&hist[d], __popc(peers));
-    }
+    if (active) atomicAdd(&hist[d], 1u);
 }
 
 // Block-wide inclusive scan of v (all 1024 threads call; wsum holds 32 words).
