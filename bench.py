@@ -238,6 +238,8 @@ def run_gpu(args, w, ws, rank, local):
                 "qpos": torch.empty(w.M, dtype=torch.int32).pin_memory()}
     e2e_steps = max(3, min(args.steps, 20))
 
+    spread = {}
+
     def time_e2e(run):
         ms = []
         for _ in range(e2e_steps):
@@ -248,6 +250,7 @@ def run_gpu(args, w, ws, rank, local):
             e1.record(stream)
             torch.cuda.synchronize()
             ms.append(e0.elapsed_time(e1))
+        spread[run] = [round(float(v), 4) for v in (np.min(ms), np.median(ms), np.max(ms))]
         return float(np.mean(ms))
 
     # eager: the calls one by one from Python
@@ -265,6 +268,7 @@ def run_gpu(args, w, ws, rank, local):
     pipelined.replay()
     torch.cuda.synchronize()
     pipe_mean = time_e2e(pipelined.replay)
+    pipe_spread = spread[pipelined.replay]
     cs.cs_sync_status()
     e2e_mean = max_over_ranks(pipe_mean, dev)
     graph_mean = max_over_ranks(graph_mean, dev)
@@ -287,6 +291,8 @@ def run_gpu(args, w, ws, rank, local):
         "e2e": {"value": round(replica_throughput(w.t_vis, e2e_mean, ws), 1), "unit": UNIT,
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "ms_per_step": round(e2e_mean, 4),
+                "ms_min_median_max": pipe_spread,
+                "steps": e2e_steps,
                 "path": "PipelinedQuery.replay (copies and kernels overlapped by layer group, "
                         "one CUDA graph)",
                 "graph_value": round(replica_throughput(w.t_vis, graph_mean, ws), 1),
