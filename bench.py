@@ -165,8 +165,12 @@ def run_gpu(args, w, ws, rank, local):
         x["k"].copy_(pristine)
         flush.zero_()
         ev[0].record(stream)
-        cs.cs_rebase_and_score(x["k"], pl, pg, fresh, w.score_layer, w.cand0, score_out=q.score,
-                               theta=w.theta, sections=w.sections)
+        if args.no_fuse:
+            cs.cs_rebase_keys(x["k"], pl, pg, theta=w.theta, sections=w.sections)
+            cs.cs_score_deviation(fresh, x["k"][w.score_layer, cand], out=q.score)
+        else:
+            cs.cs_rebase_and_score(x["k"], pl, pg, fresh, w.score_layer, w.cand0,
+                                   score_out=q.score, theta=w.theta, sections=w.sections)
         ev[1].record(stream)
         cs.cs_select_topk(q.score, w.k, w.cand0, out=q.qpos[:w.k])
         ev[2].record(stream)
@@ -174,7 +178,7 @@ def run_gpu(args, w, ws, rank, local):
         ev[3].record(stream)
 
     # the library fuses re-base and score into one launch for these shapes
-    fused = w.dtype == "bf16" and w.hkv in (1, 2, 4)
+    fused = w.dtype == "bf16" and w.hkv in (1, 2, 4) and not args.no_fuse
     launches_per_step = 3 if fused else 4
     for _ in range(args.warmup):
         one_step([torch.cuda.Event(enable_timing=True) for _ in range(4)])
@@ -397,6 +401,9 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-fuse", action="store_true",
+                    help="run re-base and score as two calls (the standalone score kernel), "
+                         "not the fused cs_rebase_and_score launch")
     ap.add_argument("--cpu-layers", type=int, default=2)
     args = ap.parse_args()
     w = W.CONFIGS[args.workload]
