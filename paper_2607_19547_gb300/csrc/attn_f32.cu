@@ -11,6 +11,8 @@ namespace {
 constexpr int kWarps = 8;
 
 __global__ void __launch_bounds__(kWarps * 32) attn_f32_kernel(AttnArgs a) {
+    pdl_wait();   // inputs may come from the previous kernel of the stream
+    pdl_trigger();
     const int lane = threadIdx.x & 31;
     const long long wid = static_cast<long long>(blockIdx.x) * kWarps + (threadIdx.x >> 5);
     const long long total = static_cast<long long>(a.n_layers) * a.M * a.hq;
@@ -73,8 +75,7 @@ cudaError_t launch_attn_f32(const AttnArgs &a, cudaStream_t s) {
     const long long warps = static_cast<long long>(a.n_layers) * a.M * a.hq;
     if (warps == 0) return cudaSuccess;
     const long long blocks = (warps + kWarps - 1) / kWarps;
-    attn_f32_kernel<<<static_cast<unsigned>(blocks), kWarps * 32, 0, s>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(attn_f32_kernel, dim3(static_cast<unsigned>(blocks)), dim3(kWarps * 32), 0, s, a);
 }
 
 }  // namespace cs

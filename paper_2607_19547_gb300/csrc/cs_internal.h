@@ -24,6 +24,30 @@ cs_status cuda_fail(cudaError_t e, const char *what);
 
 inline bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+// Launches `kernel` with programmatic stream serialization: it may start while the
+// previous kernel in `s` is still running.  A kernel launched this way calls
+// pdl_wait() (cs_device.cuh) before it reads global memory that an earlier kernel
+// may write, so only its launch and set-up overlap the earlier kernel's tail, and
+// pdl_trigger() right after, so the next kernel's CTAs may take SMs as this one's
+// finish.  Works inside stream capture.  The bf16 attention is launched normally:
+// the wait made each of its CTAs start its first loads later (about 4.5 us per
+// step at 4x1024), more than the overlap gained.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t s, Args &&...args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
 // ---- re-base (rebase.cu) ---------------------------------------------------
 struct RebaseArgs {
     const void *k_in;

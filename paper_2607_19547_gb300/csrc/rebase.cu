@@ -354,6 +354,8 @@ __device__ __forceinline__ void stream_slices(const __nv_bfloat16 *src, __nv_bfl
 // is shifts); HKV == 0: any head count, TB as passed.
 template <int HKV>
 __global__ void __launch_bounds__(kThreads, 4) rebase_bf16_kernel(RebaseArgs a, int TB_arg, int l_per_cta) {
+    pdl_wait();   // inputs may come from the previous kernel of the stream
+    pdl_trigger();
     const int hkv = HKV > 0 ? HKV : a.hkv;
     const int TB = HKV > 0 ? 8 / HKV : TB_arg;
     __shared__ float4 tab[kMaxTokensBf16 * 64];
@@ -420,6 +422,8 @@ __global__ void __launch_bounds__(kThreads, 4) rebase_bf16_kernel(RebaseArgs a, 
 
 // fp32: 16 threads per 128-element row, each owning 4 frequency pairs.
 __global__ void __launch_bounds__(kThreads) rebase_f32_kernel(RebaseArgs a, int layers_per_cta) {
+    pdl_wait();   // inputs may come from the previous kernel of the stream
+    pdl_trigger();
     __shared__ float4 tab[kMaxTokensPerCta * 64];
     __shared__ int s_delta[kMaxTokensPerCta][3];
     const int TB = max(1, (kMaxTokensPerCta / 2) / a.hkv);
@@ -487,17 +491,14 @@ cudaError_t launch_rebase(const RebaseArgs &a, cs_dtype dt, cudaStream_t s) {
                                                (a.n_layers + slots - 1) / slots);
         const int l_per_cta = (a.n_layers + groups - 1) / groups;
         dim3 grid(blocks, (a.n_layers + l_per_cta - 1) / l_per_cta);
-        switch (a.hkv) {
-            case 1: rebase_bf16_kernel<1><<<grid, kThreads, 0, s>>>(a, TB, l_per_cta); break;
-            case 2: rebase_bf16_kernel<2><<<grid, kThreads, 0, s>>>(a, TB, l_per_cta); break;
-            case 4: rebase_bf16_kernel<4><<<grid, kThreads, 0, s>>>(a, TB, l_per_cta); break;
-            default: rebase_bf16_kernel<0><<<grid, kThreads, 0, s>>>(a, TB, l_per_cta); break;
-        }
+        auto *kern = a.hkv == 1 ? rebase_bf16_kernel<1> : a.hkv == 2 ? rebase_bf16_kernel<2>
+                   : a.hkv == 4 ? rebase_bf16_kernel<4> : rebase_bf16_kernel<0>;
+        return launch_pdl(kern, grid, dim3(kThreads), 0, s, a, TB, l_per_cta);
     } else {
         const int TB = a.hkv >= kMaxTokensPerCta / 2 ? 1 : (kMaxTokensPerCta / 2) / a.hkv;
         const int layers_per_cta = 4;
         dim3 grid((a.T + TB - 1) / TB, (a.n_layers + layers_per_cta - 1) / layers_per_cta);
-        rebase_f32_kernel<<<grid, kThreads, 0, s>>>(a, layers_per_cta);
+        return launch_pdl(rebase_f32_kernel, grid, dim3(kThreads), 0, s, a, layers_per_cta);
     }
     return cudaGetLastError();
 }

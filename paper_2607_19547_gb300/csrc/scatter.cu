@@ -21,6 +21,8 @@ __global__ void __launch_bounds__(kThreads)
 scatter_kernel(uint4 *__restrict__ cache, const uint4 *__restrict__ rows, int n_layers, int T,
                long long cache_stride16, int n_rows, long long rows_stride16, int row16,
                const int *__restrict__ idx, unsigned int *status) {
+    pdl_wait();   // inputs may come from the previous kernel of the stream
+    pdl_trigger();
     const int lane = threadIdx.x & 31;
     const long long total = static_cast<long long>(n_layers) * n_rows;
     for (long long w = static_cast<long long>(blockIdx.x) * kWarps + (threadIdx.x >> 5); w < total;
@@ -50,10 +52,9 @@ cudaError_t launch_scatter(void *cache, const void *rows, int n_layers, int T, l
     if (e != cudaSuccess) return e;
     const long long want = (warps + kWarps - 1) / kWarps;
     const int grid = static_cast<int>(std::min<long long>(want, static_cast<long long>(sms) * 16));
-    scatter_kernel<<<grid, kThreads, 0, s>>>(static_cast<uint4 *>(cache), static_cast<const uint4 *>(rows),
-                                              n_layers, T, cache_stride16, n_rows, rows_stride16, row16,
-                                              idx, status);
-    return cudaGetLastError();
+    return launch_pdl(scatter_kernel, dim3(grid), dim3(kThreads), 0, s, static_cast<uint4 *>(cache),
+                      static_cast<const uint4 *>(rows), n_layers, T, cache_stride16, n_rows,
+                      rows_stride16, row16, idx, status);
 }
 
 }  // namespace cs

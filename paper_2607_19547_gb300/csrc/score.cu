@@ -49,6 +49,8 @@ template <typename T, int NJ>
 __global__ void __launch_bounds__(kWarpsPerCta * 32)
 score_kernel(const T *__restrict__ fresh, const T *__restrict__ cached, int n, int nblocks,
              long long fs, long long cst, float *__restrict__ out) {
+    pdl_wait();   // inputs may come from the previous kernel of the stream
+    pdl_trigger();
     const int lane = threadIdx.x & 31;
     const int row = blockIdx.x * kWarpsPerCta + (threadIdx.x >> 5);
     if (row >= n) return;
@@ -88,10 +90,10 @@ cudaError_t launch_typed(const void *fresh, const void *cached, int n, int E, lo
     const T *f = static_cast<const T *>(fresh);
     const T *c = static_cast<const T *>(cached);
     switch (NJ) {
-        case 1: score_kernel<T, 1><<<grid, kWarpsPerCta * 32, 0, s>>>(f, c, n, nblocks, fs, cst, out); break;
-        case 2: score_kernel<T, 2><<<grid, kWarpsPerCta * 32, 0, s>>>(f, c, n, nblocks, fs, cst, out); break;
-        case 4: score_kernel<T, 4><<<grid, kWarpsPerCta * 32, 0, s>>>(f, c, n, nblocks, fs, cst, out); break;
-        case 8: score_kernel<T, 8><<<grid, kWarpsPerCta * 32, 0, s>>>(f, c, n, nblocks, fs, cst, out); break;
+        case 1: return launch_pdl(score_kernel<T, 1>, grid, dim3(kWarpsPerCta * 32), 0, s, f, c, n, nblocks, fs, cst, out);
+        case 2: return launch_pdl(score_kernel<T, 2>, grid, dim3(kWarpsPerCta * 32), 0, s, f, c, n, nblocks, fs, cst, out);
+        case 4: return launch_pdl(score_kernel<T, 4>, grid, dim3(kWarpsPerCta * 32), 0, s, f, c, n, nblocks, fs, cst, out);
+        case 8: return launch_pdl(score_kernel<T, 8>, grid, dim3(kWarpsPerCta * 32), 0, s, f, c, n, nblocks, fs, cst, out);
         default: return cudaErrorInvalidValue;
     }
     return cudaGetLastError();

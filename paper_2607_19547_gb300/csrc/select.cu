@@ -67,6 +67,8 @@ template <int KPT>
 __global__ void __launch_bounds__(kThreads, 1)
 select_kernel(const uint32_t *__restrict__ score, int n, int k, int idx_base, int per,
               int *__restrict__ out) {
+    pdl_wait();   // inputs may come from the previous kernel of the stream
+    pdl_trigger();
     __shared__ uint32_t hist[kBins];
     __shared__ unsigned long long wsum[kWarps];
     __shared__ uint32_t s_digit, s_krem;
@@ -198,11 +200,12 @@ cudaError_t launch_select(const float *score, int n, int k, int idx_base, int *o
     const uint32_t *keys = reinterpret_cast<const uint32_t *>(score);
     const int per = (n + kThreads - 1) / kThreads;
     if (per <= 4) {
-        select_kernel<4><<<1, kThreads, 0, s>>>(keys, n, k, idx_base, 4, out);
+        return launch_pdl(select_kernel<4>, dim3(1), dim3(kThreads), 0, s, keys, n, k, idx_base, 4, out);
     } else if (per <= kRegKeys) {
-        select_kernel<kRegKeys><<<1, kThreads, 0, s>>>(keys, n, k, idx_base, kRegKeys, out);
+        return launch_pdl(select_kernel<kRegKeys>, dim3(1), dim3(kThreads), 0, s, keys, n, k, idx_base,
+                          kRegKeys, out);
     } else {
-        select_kernel<0><<<1, kThreads, 0, s>>>(keys, n, k, idx_base, per, out);
+        return launch_pdl(select_kernel<0>, dim3(1), dim3(kThreads), 0, s, keys, n, k, idx_base, per, out);
     }
     return cudaGetLastError();
 }
