@@ -24,7 +24,9 @@
 //               owns key columns [64h, 64h+64) of every S block and output
 //               dims [64h, 64h+64) of O; thread = one TMEM lane = one query
 //               row.  Reads its half of S_j, masks, exchanges the half-row
-//               maxima through shared memory (one named barrier per block),
+//               maxima through shared memory with the warp that holds the
+//               other half of the same 32 rows (a 64-thread named barrier per
+//               block; the four row quarters run independently),
 //               updates the running max (rescaling its half of O in TMEM only
 //               when the max grows by more than 2^8), writes its half of
 //               P_j = exp2(...) as bf16 over S_j's TMEM columns, and finally
@@ -139,10 +141,6 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
     decode_item(p, blockIdx.x, l, g, qt);
     const int r0 = qt * p.tok;
     const int r_last = min(p.M, r0 + p.tok) - 1;
-    const int qmin = clamp_pos(p.qpos[r0], p.T);
-    const int kmax = clamp_pos(p.qpos[r_last], p.T);
-    const int nb = kmax / kBlockN + 1;
-    const int mask_from = qmin / kBlockN;
     const uint32_t q_bytes = static_cast<uint32_t>(p.tok * p.G) * 256u;   // both 64-column halves
 
     if (warp == 0) {
@@ -191,6 +189,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
         }
         fence_proxy_async_smem();
     }
+    // the positions are read only now: a release fence above (the barrier-init fence)
+    // would otherwise wait for these global loads before the Q and K copies go out
+    const int qmin = clamp_pos(p.qpos[r0], p.T);
+    const int kmax = clamp_pos(p.qpos[r_last], p.T);
+    const int nb = kmax / kBlockN + 1;
+    const int mask_from = qmin / kBlockN;
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -309,8 +313,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
         float m_run = -INFINITY, l_run = 0.0f;
         bool ok = true;
         // Failure handling: a thread that gives up only clears `ok`; the decision to
-        // stop is taken by all 256 softmax threads together at the exchange barrier
-        // (barrier + OR), so neither warpgroup is ever left waiting at a barrier.
+        // stop is taken by both warps of a row quarter together at their exchange
+        // barrier (barrier + OR), so neither is ever left waiting there; a quarter that
+        // stops raises `abort`, which ends the other quarters' bounded waits, and every
+        // softmax thread then meets the others at the epilogue's barriers.
         for (int j = 0; j < nb; ++j) {
             const int b = j % kSBufs;
             if (ok) {
@@ -340,7 +346,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
                 }
                 slot[half * 128 + m] = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
             }
-            if (named_bar_red_or(1, 256, !ok)) {
+            // the two warps that own a row's halves (same TMEM lane quarter) meet here;
+            // the four pairs run independently of one another
+            if (named_bar_red_or(2 + qw, 64, !ok)) {
                 ok = false;
                 *abort = 1;
                 break;
