@@ -104,6 +104,39 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     return r;
 }
 
+// One warp's 64-column half of an S block from TMEM (its lane = its row), with the
+// causal mask applied on blocks that reach past the row's position: columns above
+// `lim` become -inf.
+__device__ __forceinline__ void load_s_half(uint32_t taddr, bool diag, int lim, float (&s)[64]) {
+    uint32_t sr[64];
+    tmem_ld64(taddr, sr);
+#pragma unroll
+    for (int c = 0; c < 64; ++c) s[c] = __uint_as_float(sr[c]);
+    if (diag) {
+#pragma unroll
+        for (int c = 0; c < 64; ++c)
+            if (c > lim) s[c] = -INFINITY;
+    }
+}
+
+// P = exp2(s * scale * log2(e) - m) for 64 columns, packed as bf16 pairs; returns the
+// fp32 sum of the 64 weights (affine step and sum in fp32x2).
+__device__ __forceinline__ float exp_pack(const float (&s)[64], float scale_log2, float m,
+                                          uint32_t (&pk)[32]) {
+    const float2 sc2 = make_float2(scale_log2, scale_log2);
+    const float2 nm2 = make_float2(-m, -m);
+    float2 psum = make_float2(0.0f, 0.0f);
+#pragma unroll
+    for (int e = 0; e < 32; ++e) {
+        const float2 tt = __ffma2_rn(make_float2(s[2 * e], s[2 * e + 1]), sc2, nm2);
+        const float2 pe = make_float2(__uint_as_float(ex2_approx(tt.x)),
+                                      __uint_as_float(ex2_approx(tt.y)));
+        psum = __fadd2_rn(psum, pe);
+        pk[e] = pack_bf16x2(pe.x, pe.y);
+    }
+    return psum.x + psum.y;
+}
+
 // Tile coordinates of work item `item`.  CTAs launched together should share
 // a (layer, kv head) so its K/V blocks are read from HBM once and then hit in
 // L2; to keep the tail short the heavier half of the query tiles (selected
@@ -324,63 +357,64 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
                                                     p.status, kSiteAttnSoftmax, kWaitLimitNs);
                 ok = __all_sync(0xFFFFFFFFu, w_ok);
             }
-            float s[64];
             float *slot = xchg + (j & 1) * 256;
+            const uint32_t s_addr = lane_base + b * kBlockN + col0;
+            const bool diag = j >= mask_from;
+            const int lim = qp - j * kBlockN - col0;
+            float psum = 0.0f;
+            uint32_t pk[32];
+            bool grow = true;   // the first block always sets the running max
             if (ok) {
                 tc_fence_after();
-                uint32_t sr[64];
-                tmem_ld64(lane_base + b * kBlockN + col0, sr);
-#pragma unroll
-                for (int c = 0; c < 64; ++c) s[c] = __uint_as_float(sr[c]);
-                if (j >= mask_from) {
-                    const int lim = qp - j * kBlockN - col0;
-#pragma unroll
-                    for (int c = 0; c < 64; ++c)
-                        if (c > lim) s[c] = -INFINITY;
-                }
+                float s[64];
+                load_s_half(s_addr, diag, lim, s);
                 float mx4[4] = {s[0], s[1], s[2], s[3]};
 #pragma unroll
                 for (int c = 4; c < 64; c += 4) {
 #pragma unroll
                     for (int q = 0; q < 4; ++q) mx4[q] = fmaxf(mx4[q], s[c + q]);
                 }
-                slot[half * 128 + m] = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
+                const float mxh = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
+                slot[half * 128 + m] = mxh;
+                if (j > 0) {
+                    // this half of P_j with the running max of the earlier blocks, which
+                    // the row keeps unless its maximum grows by more than 2^8 in either
+                    // half (checked at the barrier below; then P_j is recomputed), so the
+                    // exponentials need not wait for the other half's maximum
+                    grow = mxh * p.scale_log2 > m_run + 8.0f;
+                    psum = exp_pack(s, p.scale_log2, m_run, pk);
+                }
             }
             // the two warps that own a row's halves (same TMEM lane quarter) meet here;
-            // the four pairs run independently of one another
-            if (named_bar_red_or(2 + qw, 64, !ok)) {
-                ok = false;
-                *abort = 1;
-                break;
-            }
-            const float mx = fmaxf(slot[m], slot[128 + m]);
-            const float mx2 = mx * p.scale_log2;
-            const bool grow = (m_run == -INFINITY) || (mx2 > m_run + 8.0f);
+            // the four pairs run independently of one another.  A failure or a raised
+            // maximum in either warp takes both through the exchange.
+            bool rescale = false;
             float alpha = 1.0f;
-            if (grow) {
-                alpha = exp2f(m_run - mx2);   // 0 on the first block
-                l_run *= alpha;
-                m_run = mx2;
+            if (named_bar_red_or(2 + qw, 64, !ok || grow)) {
+                if (named_bar_red_or(2 + qw, 64, !ok)) {
+                    ok = false;
+                    *abort = 1;
+                    break;
+                }
+                const float mx2 = fmaxf(slot[m], slot[128 + m]) * p.scale_log2;
+                const bool g = (m_run == -INFINITY) || (mx2 > m_run + 8.0f);
+                if (g) {
+                    alpha = exp2f(m_run - mx2);   // 0 on the first block
+                    l_run *= alpha;
+                    m_run = mx2;
+                }
+                rescale = j > 0 && __any_sync(0xFFFFFFFFu, g);
+                // S_j is still in TMEM (P_j has not been written over it yet)
+                float s[64];
+                load_s_half(s_addr, diag, lim, s);
+                psum = exp_pack(s, p.scale_log2, m_run, pk);
             }
-            // this half of P_j = exp2(s * scale * log2(e) - m_run), packed bf16 into
-            // columns [32h, 32h+32) of S_j's buffer; affine step and sum in fp32x2
-            const float2 sc2 = make_float2(p.scale_log2, p.scale_log2);
-            const float2 nm2 = make_float2(-m_run, -m_run);
-            float2 psum = make_float2(0.0f, 0.0f);
-            uint32_t pk[32];
-#pragma unroll
-            for (int e = 0; e < 32; ++e) {
-                const float2 tt = __ffma2_rn(make_float2(s[2 * e], s[2 * e + 1]), sc2, nm2);
-                const float2 pe = make_float2(__uint_as_float(ex2_approx(tt.x)),
-                                              __uint_as_float(ex2_approx(tt.y)));
-                psum = __fadd2_rn(psum, pe);
-                pk[e] = pack_bf16x2(pe.x, pe.y);
-            }
+            // packed bf16 into columns [32h, 32h+32) of S_j's buffer
             tmem_st32(lane_base + b * kBlockN + 32 * half, pk);
-            l_run += psum.x + psum.y;
+            l_run += psum;
             // rescale this half of O when any row of the warp raised its max
             // (O holds PV_0 .. PV_{j-1})
-            if (j > 0 && __any_sync(0xFFFFFFFFu, grow)) {
+            if (rescale) {
                 const bool o_ok = mbar_wait_bounded(&bars->pv_done[(j - 1) % kSBufs],
                                                     ((j - 1) / kSBufs) & 1, abort, p.status,
                                                     kSiteAttnSoftmax, kWaitLimitNs);
