@@ -81,6 +81,22 @@ def test_bf16_large_logits_rescale(cslib):
                    v.to(torch.bfloat16), qpos, "bf16")
 
 
+def test_bf16_max_grows_in_one_half(cslib):
+    """One large key in the first half of block 1's columns, a larger one in the second half of
+    block 2's: the running maximum of the rows that see them rises by more than 2^8 in one
+    64-column half only, so both halves of those rows must take the new maximum together."""
+    L, T, Hq, Hkv = 1, 512, 8, 1
+    q = torch.full((L, 16, Hq, 128), 0.5, device="cuda")
+    k = _rand((L, T, Hkv, 128), 15, torch.float32) * 0.1
+    v = _rand((L, T, Hkv, 128), 16, torch.float32)
+    k[0, 150] = 1.5          # block 1, column 22: scores +8.5 (x log2(e) > 8)
+    k[0, 330] = 3.0          # block 2, column 74: scores +17
+    qpos = np.array([100, 149, 150, 151, 200, 255, 256, 300, 329, 330, 331, 383, 384, 400,
+                     450, 511], np.int32)
+    _run_and_check(cslib, q.to(torch.bfloat16), k.to(torch.bfloat16), v.to(torch.bfloat16),
+                   qpos, "bf16")
+
+
 def test_qwen3b_4x1024_all_rows(cslib):
     w = W.CONFIGS["qwen3b_4x1024"]
     x = W.make_inputs(w, seed=0, device="cuda")
