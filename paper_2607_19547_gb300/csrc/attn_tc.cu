@@ -23,15 +23,18 @@
 //   warps 2-9   softmax, two warpgroups: warpgroup h (warps 2+4h .. 5+4h)
 //               owns key columns [64h, 64h+64) of every S block and output
 //               dims [64h, 64h+64) of O; thread = one TMEM lane = one query
-//               row.  Reads its half of S_j, masks, exchanges the half-row
-//               maxima through shared memory with the warp that holds the
-//               other half of the same 32 rows (a 64-thread named barrier per
-//               block; the four row quarters run independently),
-//               updates the running max (rescaling its half of O in TMEM only
-//               when the max grows by more than 2^8), writes its half of
-//               P_j = exp2(...) as bf16 over S_j's TMEM columns, and finally
-//               normalises its half of O into the Q tile's shared memory (idle
-//               after the last S), from where two TMA stores write whole rows.
+//               row.  Reads its half of S_j, masks, takes the half-row maxima
+//               and computes its half of P_j = exp2(...) with the running max
+//               of the earlier blocks, then meets the warp that holds the
+//               other half of the same 32 rows (a 64-thread named barrier with
+//               an OR per block; the four row quarters run independently).
+//               The running max is raised only when it grows by more than
+//               2^8; when that happens in either half, both warps exchange
+//               their maxima through shared memory, raise it, recompute P_j
+//               from S_j and rescale their half of O in TMEM.  P_j is written
+//               as bf16 over S_j's TMEM columns.  Finally each warp normalises
+//               its half of O into the Q tile's shared memory (idle after the
+//               last S), from where two TMA stores write whole rows.
 // TMEM: S buffers at columns 0, 128, 256; O at 384.  S_j reuses the buffer
 // of P_{j-3}, so the S issuer runs up to three blocks ahead of the softmax.
 // Every mbarrier wait is bounded; on a timeout the CTA records
