@@ -145,6 +145,41 @@ class GraphedQuery:
         return self.h2d, self.d2h
 
 
+def plan_layer_groups(n_layers: int, score_layer: int, group_layers: int = 4, bounds=None):
+    """Layer groups of a pipelined query, as (first, end) pairs covering [0, n_layers).
+
+    By default: a short first group that reaches the score layer (the pipeline waits for its
+    upload, so the selection runs as early as possible), groups of group_layers, and a short
+    last group of 2 layers (its compute and download trail the last upload).  bounds, when
+    given, are the group boundaries themselves: they must rise strictly from 0 to n_layers,
+    and the first group must hold the score layer (every group's attention reads the
+    selection that the score layer's group makes)."""
+    if n_layers < 1:
+        raise ValueError("n_layers must be at least 1")
+    if not 0 <= score_layer < n_layers:
+        raise ValueError("score_layer must be a layer of the cache")
+    if bounds is None:
+        if group_layers < 1:
+            raise ValueError("group_layers must be at least 1")
+        L = n_layers
+        lead, tail = min(L, max(2, score_layer + 1)), 2
+        bounds = [0, lead]
+        while bounds[-1] + group_layers < L - tail:
+            bounds.append(bounds[-1] + group_layers)
+        if L - tail > bounds[-1]:
+            bounds.append(L - tail)
+        if L > bounds[-1]:
+            bounds.append(L)
+    bounds = [int(x) for x in bounds]
+    if (len(bounds) < 2 or bounds[0] != 0 or bounds[-1] != n_layers
+            or any(b <= a for a, b in zip(bounds[:-1], bounds[1:]))):
+        raise ValueError("bounds must rise strictly from 0 to n_layers")
+    if not score_layer < bounds[1]:
+        # every group's attention reads the selection, which the score layer's group makes
+        raise ValueError("the first group must hold the score layer")
+    return list(zip(bounds[:-1], bounds[1:]))
+
+
 class PipelinedQuery:
     """An end-to-end query from host buffers with the copies and the kernels overlapped layer
     group by layer group, captured as one CUDA graph.
@@ -164,25 +199,7 @@ class PipelinedQuery:
             raise ValueError(f"policy must be one of {POLICIES}")
         s = query.shape
         self.query, self.host, self.dev, self.out_host = query, host, dev, out_host
-        L = s.n_layers
-        if bounds is None:
-            # a short first group that reaches the score layer (the pipeline waits for its
-            # upload; the selection runs as early as possible), groups of group_layers, and
-            # a short last group (its compute and download trail the last upload)
-            lead, tail = min(L, max(2, s.score_layer + 1)), 2
-            bounds = [0, lead]
-            while bounds[-1] + group_layers < L - tail:
-                bounds.append(bounds[-1] + group_layers)
-            if L - tail > bounds[-1]:
-                bounds.append(L - tail)
-            if L > bounds[-1]:
-                bounds.append(L)
-        bounds = list(bounds)
-        if bounds[0] != 0 or bounds[-1] != L or any(b <= a for a, b in zip(bounds[:-1], bounds[1:])):
-            raise ValueError("bounds must rise strictly from 0 to n_layers")
-        if not any(a <= s.score_layer < b for a, b in zip(bounds[:-1], bounds[1:])):
-            raise ValueError("the score layer must lie in a group")
-        self.groups = list(zip(bounds[:-1], bounds[1:]))
+        self.groups = plan_layer_groups(s.n_layers, s.score_layer, group_layers, bounds)
         device = dev["k"].device
         self.s_in, self.s_c, self.s_out = (torch.cuda.Stream(device=device) for _ in range(3))
         self.h2d = sum(host[n].numel() * host[n].element_size() for n in ("k", "v", "q", "k_fresh"))

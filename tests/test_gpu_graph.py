@@ -71,10 +71,11 @@ def test_graph_replay_equals_eager(cslib, name):
         assert torch.equal(got["o"], eager["o"])
 
 
-@pytest.mark.parametrize("name,policy,group", [("tiny_f32", "3axis", 6), ("qwen3b_4x1024", "3axis", 6),
-                                               ("qwen3b_4x1024", "scalar1d", 5),
-                                               ("qwen3b_4x1024", "naive", 36)])
-def test_pipelined_query_equals_eager(cslib, name, policy, group):
+@pytest.mark.parametrize("name,policy,group,bounds", [
+    ("tiny_f32", "3axis", 6, None), ("qwen3b_4x1024", "3axis", 6, None),
+    ("qwen3b_4x1024", "scalar1d", 5, None), ("qwen3b_4x1024", "naive", 36, None),
+    ("qwen3b_4x1024", "3axis", 4, [0, 2, 3, 20, 35, 36])])
+def test_pipelined_query_equals_eager(cslib, name, policy, group, bounds):
     """Uploads, kernels and downloads overlapped layer group by layer group (one graph) give the
     eager query's result bit for bit."""
     from paper_2607_19547_gb300.pipeline import PipelinedQuery
@@ -87,7 +88,7 @@ def test_pipelined_query_equals_eager(cslib, name, policy, group):
     torch.cuda.synchronize()
     qp = ComposedQuery(shape, w.torch_dtype)
     got = _out_host(qp, w)
-    pq = PipelinedQuery(qp, host, dev, got, group_layers=group, policy=policy)
+    pq = PipelinedQuery(qp, host, dev, got, group_layers=group, policy=policy, bounds=bounds)
     for _ in range(2):
         for t in got.values():
             t.zero_()
