@@ -163,7 +163,8 @@ cs_status cs_select_topk(const float *score, int n, int k, int32_t idx_base, int
  *   j = 0 .. qpos[r]  (causal in global sequence order, the row's own key included),
  *   G = n_q_heads / n_kv_heads (grouped-query attention).
  *
- *   q, o     [n_layers][M][n_q_heads][head_dim], contiguous
+ *   q, o     [n_layers][M][n_q_heads][head_dim], contiguous; o may be q itself
+ *            but must not overlap k or v (CS_ERR_INVALID_ARG)
  *   k, v     [n_layers][T][n_kv_heads][head_dim] with layer stride kv_layer_stride
  *   qpos     int32 [M], strictly ascending, 0 <= qpos[r] < T (checked on the
  *            device; a violation yields CS_ERR_DEVICE_ARG at cs_sync_status and

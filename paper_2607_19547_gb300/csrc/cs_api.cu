@@ -323,6 +323,18 @@ cs_status cs_repair_attention(const void *q, const void *k, const void *v, void 
         return fail(CS_ERR_INVALID_ARG, "q, k, v, o must be 16-byte aligned (and the layer stride)");
     if (dtype == CS_DTYPE_BF16 && static_cast<long long>(M) * n_q_heads > 0x7FFFFFFFll)
         return fail(CS_ERR_UNSUPPORTED, "M * n_q_heads too large");
+    {
+        // o is written while other CTAs still read k and v (each o element is written by
+        // the CTA that read the same element of q, so o == q is allowed)
+        const long long kv_span =
+            ((n_layers - 1) * kv_layer_stride + static_cast<long long>(T) * n_kv_heads * head_dim) * esz;
+        const long long o_span = static_cast<long long>(n_layers) * M * n_q_heads * head_dim * esz;
+        const char *oc = static_cast<const char *>(o);
+        const char *kc = static_cast<const char *>(k);
+        const char *vc = static_cast<const char *>(v);
+        if ((oc < kc + kv_span && kc < oc + o_span) || (oc < vc + kv_span && vc < oc + o_span))
+            return fail(CS_ERR_INVALID_ARG, "o overlaps k or v");
+    }
     unsigned int *status = status_word();
     if (status == nullptr) return CS_ERR_CUDA;
     AttnArgs a;

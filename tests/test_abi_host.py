@@ -130,6 +130,8 @@ def test_attention_rejects_bad_arguments(cslib):
     assert call(T=0, st=0) == cslib.CS_ERR_INVALID_ARG
     assert call(qpos=None) == cslib.CS_ERR_INVALID_ARG
     assert call(o=FAKE + 4) == cslib.CS_ERR_INVALID_ARG
+    assert call() == cslib.CS_ERR_INVALID_ARG           # o over k and v
+    assert "overlaps" in cslib.cs_last_error_detail()
     assert call(Hq=256, Hkv=1) == cslib.CS_ERR_UNSUPPORTED
     assert call(M=0, q=None, o=None) == cslib.CS_OK
 
