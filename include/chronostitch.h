@@ -150,7 +150,7 @@ cs_status cs_rebase_and_score(const void *k_in, void *k_out, cs_dtype dtype, int
  * (rho_bp*n + 9999)/10000.
  *
  *   score    fp32 [n], device memory;   0 <= k <= n;   idx_base + n <= INT32_MAX
- *   out_idx  int32 [k], device memory
+ *   out_idx  int32 [k], device memory, not overlapping score (CS_ERR_INVALID_ARG)
  */
 cs_status cs_select_topk(const float *score, int n, int k, int32_t idx_base, int32_t *out_idx,
                          void *stream);

@@ -255,6 +255,13 @@ cs_status cs_select_topk(const float *score, int n, int k, int32_t idx_base, int
         return fail(CS_ERR_INVALID_ARG, "idx_base + n must stay within int32");
     if (k == 0) return CS_OK;
     if (score == nullptr || out_idx == nullptr) return fail(CS_ERR_INVALID_ARG, "NULL pointer");
+    {
+        // the indices are written while scores may still be read (large n re-reads them)
+        const char *sc = reinterpret_cast<const char *>(score);
+        const char *oc = reinterpret_cast<const char *>(out_idx);
+        if (oc < sc + 4ll * n && sc < oc + 4ll * k)
+            return fail(CS_ERR_INVALID_ARG, "out_idx overlaps score");
+    }
     const cudaError_t e = launch_select(score, n, k, idx_base, out_idx, as_stream(stream));
     if (e != cudaSuccess) return cuda_fail(e, "select launch");
     return CS_OK;

@@ -110,6 +110,8 @@ def test_select_rejects_bad_arguments(cslib):
     assert L.cs_select_topk(FAKE, 10, 3, -1, FAKE, None) == cslib.CS_ERR_INVALID_ARG
     assert L.cs_select_topk(None, 10, 3, 0, FAKE, None) == cslib.CS_ERR_INVALID_ARG
     assert L.cs_select_topk(None, 10, 0, 0, None, None) == cslib.CS_OK
+    assert L.cs_select_topk(FAKE, 10, 3, 0, FAKE + 16, None) == cslib.CS_ERR_INVALID_ARG
+    assert "overlaps" in cslib.cs_last_error_detail()
 
 
 def test_attention_rejects_bad_arguments(cslib):
