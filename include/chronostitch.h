@@ -109,7 +109,7 @@ cs_status cs_rebase_keys(const void *k_in, void *k_out, cs_dtype dtype, int n_la
  *   k_fresh   row t at k_fresh + t*fresh_row_stride, E contiguous elements
  *   k_cached  row t at k_cached + t*cached_row_stride (e.g. the re-based layer-1
  *             rows of the composed cache: stride n_kv_heads*head_dim)
- *   score_out fp32 [n]
+ *   score_out fp32 [n], not overlapping either key array (CS_ERR_INVALID_ARG)
  */
 cs_status cs_score_deviation(const void *k_fresh, const void *k_cached, cs_dtype dtype, int n,
                              int n_kv_heads, int head_dim, int64_t fresh_row_stride,
@@ -128,7 +128,7 @@ cs_status cs_score_deviation(const void *k_fresh, const void *k_cached, cs_dtype
  *   0 <= score_layer < n_layers (when n_cand > 0);  0 <= cand0,  cand0 + n_cand <= T
  *   k_fresh    row c (token cand0 + c) at k_fresh + c*fresh_row_stride, E elements,
  *              device memory, 16-byte aligned rows, not overlapping k_out
- *   score_out  fp32 [n_cand], device memory
+ *   score_out  fp32 [n_cand], device memory, not overlapping the keys or k_fresh
  * Other arguments and errors as for cs_rebase_keys and cs_score_deviation.
  */
 cs_status cs_rebase_and_score(const void *k_in, void *k_out, cs_dtype dtype, int n_layers,

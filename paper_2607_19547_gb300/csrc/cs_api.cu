@@ -104,6 +104,13 @@ const char *cs_last_error_detail(void) { return t_detail; }
 
 namespace {
 
+// [a, a + an) and [b, b + bn) (bytes) share an address
+bool overlaps(const void *a, long long an, const void *b, long long bn) {
+    const char *x = static_cast<const char *>(a);
+    const char *y = static_cast<const char *>(b);
+    return x < y + bn && y < x + an;
+}
+
 // The layer-`score_layer` score requested together with a re-base.
 struct ScoreRequest {
     int score_layer, cand0, n_cand;
@@ -151,6 +158,17 @@ cs_status rebase_impl(const void *k_in, void *k_out, cs_dtype dtype, int n_layer
             return fail(CS_ERR_INVALID_ARG, "NULL fresh keys or score output");
         if (scoring && (!aligned16(sc->fresh) || (sc->fresh_stride * esz) % 16))
             return fail(CS_ERR_INVALID_ARG, "fresh rows must start 16-byte aligned");
+        if (scoring && n_layers > 0 && T > 0) {
+            const long long out_bytes = 4ll * sc->n_cand;
+            const long long keys_bytes = ((n_layers - 1) * layer_stride + T * row) * esz;
+            const long long fresh_bytes = ((sc->n_cand - 1) * sc->fresh_stride + row) * esz;
+            if (overlaps(sc->score_out, out_bytes, k_in, keys_bytes) ||
+                overlaps(sc->score_out, out_bytes, k_out, keys_bytes) ||
+                overlaps(sc->score_out, out_bytes, sc->fresh, fresh_bytes))
+                return fail(CS_ERR_INVALID_ARG, "score_out overlaps the keys");
+            if (overlaps(sc->fresh, fresh_bytes, k_out, keys_bytes))
+                return fail(CS_ERR_INVALID_ARG, "k_fresh overlaps the re-based keys");
+        }
     }
     if (n_layers == 0 || T == 0) return CS_OK;
     if (k_in == nullptr || k_out == nullptr || pos_local == nullptr || pos_global == nullptr)
@@ -241,6 +259,9 @@ cs_status cs_score_deviation(const void *k_fresh, const void *k_cached, cs_dtype
     if (!aligned16(k_fresh) || !aligned16(k_cached) || (fresh_row_stride * esz) % 16 ||
         (cached_row_stride * esz) % 16)
         return fail(CS_ERR_INVALID_ARG, "rows must start 16-byte aligned");
+    if (overlaps(score_out, 4ll * n, k_fresh, ((n - 1) * fresh_row_stride + E) * esz) ||
+        overlaps(score_out, 4ll * n, k_cached, ((n - 1) * cached_row_stride + E) * esz))
+        return fail(CS_ERR_INVALID_ARG, "score_out overlaps the keys");
     const cudaError_t e = launch_score(k_fresh, k_cached, dtype, n, static_cast<int>(E),
                                        fresh_row_stride, cached_row_stride, score_out,
                                        as_stream(stream));

@@ -100,6 +100,8 @@ def test_score_rejects_bad_arguments(cslib):
     assert call(fs=260) == cslib.CS_ERR_INVALID_ARG         # 520-byte rows break 16 B alignment
     assert call(H=17) == cslib.CS_ERR_UNSUPPORTED
     assert call(n=0, f=None, c=None, out=None) == cslib.CS_OK
+    assert call() == cslib.CS_ERR_INVALID_ARG              # score_out over the key rows
+    assert "overlaps" in cslib.cs_last_error_detail()
 
 
 def test_select_rejects_bad_arguments(cslib):
@@ -196,4 +198,8 @@ def test_rebase_and_score_rejects_bad_arguments(cslib):
     assert call(fr=FAKE + 8) == cslib.CS_ERR_INVALID_ARG    # misaligned fresh rows
     assert call(out=None) == cslib.CS_ERR_INVALID_ARG
     assert call(D=64) == cslib.CS_ERR_UNSUPPORTED
+    assert call(out=FAKE + 64) == cslib.CS_ERR_INVALID_ARG  # score_out over the keys
+    assert "overlaps" in cslib.cs_last_error_detail()
+    assert call(fr=FAKE + 256) == cslib.CS_ERR_INVALID_ARG  # fresh rows inside the keys
+    assert "overlaps" in cslib.cs_last_error_detail()
     assert call(L=0, nc=0) == cslib.CS_OK
