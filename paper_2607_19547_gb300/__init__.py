@@ -114,9 +114,14 @@ def _dtype_code(t: torch.Tensor) -> int:
 
 
 def _need_cuda(*ts):
+    """CUDA tensors, all on the current device (the library launches there)."""
     for t in ts:
         if not (isinstance(t, torch.Tensor) and t.is_cuda):
             raise ValueError("all tensors must be CUDA tensors")
+    cur = torch.cuda.current_device()
+    for t in ts:
+        if t.device.index != cur:
+            raise ValueError(f"tensor on {t.device}, but the current device is cuda:{cur}")
 
 
 def _inner_contiguous(t: torch.Tensor, what: str):
@@ -246,9 +251,9 @@ def cs_repair_attention(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, qpos:
         raise ValueError("q must be contiguous")
     _inner_contiguous(k, "k")
     L, M, Hq, D = q.shape
-    _, T, Hkv, _ = k.shape
-    if k.shape[0] != L or k.dtype != q.dtype or v.dtype != q.dtype:
-        raise ValueError("q, k, v must share layers and dtype")
+    _, T, Hkv, Dk = k.shape
+    if k.shape[0] != L or Dk != D or k.dtype != q.dtype or v.dtype != q.dtype:
+        raise ValueError("q, k, v must share layers, head dim and dtype")
     if qpos.dtype != torch.int32 or qpos.numel() != M or not qpos.is_contiguous():
         raise ValueError("qpos must be contiguous int32 [M]")
     if out is None:

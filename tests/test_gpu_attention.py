@@ -133,6 +133,14 @@ def test_single_key_and_empty(cslib):
     assert empty.numel() == 0
 
 
+def test_binding_rejects_a_head_dim_mismatch(cslib):
+    """K and V must have Q's head dim: with one layer no stride would give the mismatch away."""
+    q = _rand((1, 4, 16, 128), 17, torch.bfloat16)
+    k = _rand((1, 64, 2, 64), 18, torch.bfloat16)
+    with pytest.raises(ValueError):
+        cslib.cs_repair_attention(q, k, k, cuda(np.array([3, 10, 20, 30], np.int32)))
+
+
 def test_bad_query_positions_are_reported(cslib):
     q = _rand((1, 4, 16, 128), 13, torch.bfloat16)
     k = _rand((1, 64, 2, 128), 14, torch.bfloat16)
