@@ -71,7 +71,7 @@ select_kernel(const uint32_t *__restrict__ score, int n, int k, int idx_base, in
     pdl_trigger();
     __shared__ uint32_t hist[kBins];
     __shared__ unsigned long long wsum[kWarps];
-    __shared__ uint32_t s_digit, s_krem;
+    __shared__ uint32_t s_digit, s_krem, s_done;
     const int tid = threadIdx.x;
 
     if (k >= n) {   // everything is selected, in index order
@@ -130,34 +130,41 @@ select_kernel(const uint32_t *__restrict__ score, int n, int k, int idx_base, in
             block_incl_scan<unsigned long long>(static_cast<unsigned long long>(hi + lo), wsum);
         const unsigned long long above = incl - (hi + lo);
         if (above < krem && incl >= krem) {
+            // the bin holding the k-th largest key; when every key left in it is taken,
+            // the remaining digits cannot change the selection and the passes stop
             if (above + hi >= krem) {
                 s_digit = static_cast<uint32_t>(kBins - 1 - 2 * tid);
                 s_krem = krem - static_cast<uint32_t>(above);
+                s_done = hi == s_krem;
             } else {
                 s_digit = static_cast<uint32_t>(kBins - 2 - 2 * tid);
                 s_krem = krem - static_cast<uint32_t>(above) - hi;
+                s_done = lo == s_krem;
             }
         }
         __syncthreads();
         prefix |= s_digit << shift;
         pmask |= dmask << shift;
         krem = s_krem;
-        __syncthreads();   // s_digit / wsum are rewritten by the next pass
+        if (s_done) break;   // uniform; nothing shared is written again before it is read
+        __syncthreads();     // s_digit / wsum are rewritten by the next pass
     }
-    // prefix = K*; krem = how many keys equal to K* are selected (lowest indices first)
+    // prefix = the resolved high bits of K* (all of K* after three passes) and pmask
+    // their mask; krem = how many keys with that prefix are selected (lowest indices first;
+    // all of them when the passes stopped early)
     const uint32_t kstar = prefix;
     uint32_t gt = 0, eq = 0;
     if (KPT > 0) {
 #pragma unroll
         for (int i = 0; i < (KPT > 0 ? KPT : 1); ++i) {
-            gt += (i < cnt && reg[i] > kstar);
-            eq += (i < cnt && reg[i] == kstar);
+            gt += (i < cnt && (reg[i] & pmask) > kstar);
+            eq += (i < cnt && (reg[i] & pmask) == kstar);
         }
     } else {
         for (int c0 = 0; c0 < cnt; c0 += 8) {   // eight loads in flight
             uint32_t kb[8];
 #pragma unroll
-            for (int u = 0; u < 8; ++u) kb[u] = c0 + u < cnt ? key_at(c0 + u) : 0u;
+            for (int u = 0; u < 8; ++u) kb[u] = c0 + u < cnt ? (key_at(c0 + u) & pmask) : 0u;
 #pragma unroll
             for (int u = 0; u < 8; ++u) {
                 gt += c0 + u < cnt && kb[u] > kstar;
@@ -173,7 +180,7 @@ select_kernel(const uint32_t *__restrict__ score, int n, int k, int idx_base, in
     if (KPT > 0) {
 #pragma unroll
         for (int i = 0; i < (KPT > 0 ? KPT : 1); ++i) {
-            const uint32_t key = reg[i];
+            const uint32_t key = reg[i] & pmask;
             if (i < cnt && (key > kstar || (key == kstar && eq_seen++ < krem)))
                 out[pos++] = idx_base + i0 + i;
         }
@@ -181,7 +188,7 @@ select_kernel(const uint32_t *__restrict__ score, int n, int k, int idx_base, in
         for (int c0 = 0; c0 < cnt; c0 += 8) {
             uint32_t kb[8];
 #pragma unroll
-            for (int u = 0; u < 8; ++u) kb[u] = c0 + u < cnt ? key_at(c0 + u) : 0u;
+            for (int u = 0; u < 8; ++u) kb[u] = c0 + u < cnt ? (key_at(c0 + u) & pmask) : 0u;
 #pragma unroll
             for (int u = 0; u < 8; ++u) {
                 const uint32_t key = kb[u];
