@@ -4,11 +4,12 @@
 // stay in L2).  Scores map to order-preserving 32-bit keys.  Thread t owns the
 // contiguous candidate range [t*per, (t+1)*per); up to 16 keys per thread stay
 // in registers, larger inputs are re-read from L2 in every pass (the histogram
-// passes read them interleaved and coalesced, eight loads in flight).  Three
+// passes read them interleaved and coalesced, eight loads in flight).  Up to three
 // MSB-first radix passes over 11-, 11- and 10-bit digits (one shared 2048-bin
 // histogram, shared-memory atomic increments) find K*, the k-th largest key, and how
 // many keys equal to K* belong to the top k (the lowest-index ones: the
-// tie-break).  One block-wide scan of the per-thread (greater, equal) counts
+// tie-break); they stop early once every key left in K*'s bin is taken, and the
+// resolved prefix of K* then stands for it.  One block-wide scan of the per-thread (greater, equal) counts
 // then gives every selected index its output position, so the output is
 // ascending without a sort.
 #include "cs_device.cuh"
