@@ -56,6 +56,23 @@ def test_bf16_group_sizes_ragged(cslib, Hq, Hkv):
     _run_and_check(cslib, q, k, v, qpos, "bf16")
 
 
+@pytest.mark.parametrize("seed", range(6))
+def test_bf16_random_shapes(cslib, seed):
+    """Seeded random shapes: GQA groups that do not divide 128 (3, 5, 6: tiles of 126, 125 and
+    126 rows with spare rows zeroed), ragged key counts, several layers, random positions."""
+    rng = np.random.default_rng(100 + seed)
+    G = [3, 5, 6, 12, 4, 1][seed]
+    Hkv = int(rng.choice([1, 2, 3]))
+    L = int(rng.integers(1, 4))
+    T = int(rng.integers(130, 900))
+    M = int(rng.integers(1, min(T, 90)))
+    q = _rand((L, M, G * Hkv, 128), 200 + seed, torch.bfloat16)
+    k = _rand((L, T, Hkv, 128), 300 + seed, torch.bfloat16)
+    v = _rand((L, T, Hkv, 128), 400 + seed, torch.bfloat16)
+    qpos = np.sort(rng.choice(T, size=M, replace=False)).astype(np.int32)
+    _run_and_check(cslib, q, k, v, qpos, "bf16")
+
+
 def test_bf16_dense_rows_and_block_edges(cslib):
     """Consecutive rows and rows on key-block boundaries (127, 128, 255, 256, ...)."""
     L, T, Hq, Hkv = 1, 700, 16, 2
