@@ -2,25 +2,30 @@
 
 One step = one composition query: re-base all layers' stored keys, score the
 candidates, select the top rho, repair-attend the selected rows over the
-composed cache (four kernel launches).  The metric is composed visual tokens
-per second: T_vis / step time.
+composed cache (three kernel launches: re-base and score are one).  The metric
+is composed visual tokens per second: T_vis / step time.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl ours|reference]
 
-Prints one JSON line (rank 0).  --impl reference times the CPU oracle on the
-host cores instead (a bounded sample of each step, scaled to the full step).
-With N > 1 (torchrun) every rank runs an independent replica of the query.
+Prints one JSON line (rank 0).  The default workload is the largest single-GPU
+configuration, qwen3b_64x1024_r15 (3B shape, 64 chunks x 1024 tokens, rho 0.15).
+--impl reference times the CPU oracle on the host cores instead: each step is a
+bounded sample of the workload (one layer of re-base, score and select over all
+candidates, attention of a seeded sample of rows), scaled to the full step by the
+work it stands for.  With N > 1 (torchrun) every rank runs an independent replica
+of the query; the reference arm runs on rank 0 only.
 """
 from __future__ import annotations
 
 import os
 
-# the CPU oracle is timed single-threaded: fix BLAS / OpenMP threads before numpy loads
+# the oracle is timed on explicit worker processes: one BLAS / OpenMP thread each
 for _v in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
     os.environ.setdefault(_v, "1")
 
 import argparse
 import json
+import platform
 import statistics
 import subprocess
 import sys
@@ -36,6 +41,8 @@ import cs_workloads as W  # noqa: E402
 
 METRIC = "composed visual tokens/sec (rebase+score+select+repair attn); % HBM / tensor peak"
 UNIT = "tokens/s"
+DATA = ("synthetic: seeded N(0,1) stored keys/values/queries, lognormal fresh-key deviation, "
+        "Qwen2.5-VL-shaped")
 
 
 def _dist_env():
@@ -71,17 +78,38 @@ def peaks():
 
 
 def profiled_traffic(kernel_file: str):
-    """dram bytes per launch recorded in a committed ncu summary (profiles/<file>), else None."""
+    """(dram bytes per launch, source note) from a committed ncu summary, or (None, why)."""
     path = os.path.join(ROOT, "profiles", kernel_file)
     if not os.path.exists(path):
-        return None
+        return None, f"no committed ncu summary profiles/{kernel_file}"
     for line in open(path):
         if line.startswith("dram_bytes_per_launch_full_workload:"):
             try:
-                return float(line.split(":", 1)[1].split()[0])
+                v = float(line.split(":", 1)[1].split()[0])
             except ValueError:
-                return None
-    return None
+                break
+            return v, (f"profiles/{kernel_file}: dram__bytes_read.sum + dram__bytes_write.sum "
+                       "of an ncu capture (not measured by this run)")
+    return None, f"profiles/{kernel_file} holds no per-launch DRAM figure"
+
+
+def cpu_model() -> str:
+    """The host CPU's model name (lscpu), else what the platform module knows."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().startswith("Model name:"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    return platform.processor() or platform.machine()
+
+
+def host_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
 
 
 class ClockSampler:
@@ -133,6 +161,17 @@ class ClockSampler:
         return {"sm_mhz": statistics.median(sm) if sm else None,
                 "sm_max_mhz": max(smax) if smax else None,
                 "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def config_of(w, ws: int) -> dict:
+    """The workload description both arms print (the same dict for the same run)."""
+    return {"workload": w.name, "layers": w.n_layers, "chunks": w.n_chunks,
+            "tokens_per_chunk": w.chunk_tokens, "T": w.T, "T_vis": w.t_vis,
+            "q_heads": w.hq, "kv_heads": w.hkv, "rho": w.rho_bp / 1e4, "k": w.k,
+            "suffix_rows": w.suffix,
+            "l2": "inputs larger than L2; also flushed between steps (256 MB write) with the "
+                  "stored keys restored, untimed",
+            "parallelism": f"{ws} independent replica(s)"}
 
 
 # ----------------------------------------------------------------------------- GPU arm
@@ -234,22 +273,30 @@ def run_gpu(args, w, ws, rank, local):
     pk = peaks()
     attn_flop = W.attention_flops(w, qpos)
     mean = per.mean(axis=0)            # ms: re-base + score + select, attention
-    rb_bytes, sc_bytes = W.rebase_bytes(w), W.score_bytes(w)
     sel_bytes = 4.0 * w.n_cand + 4.0 * w.k
     attn_tflops = attn_flop / (mean[1] / 1e3) / 1e12
-    traffic = profiled_traffic(f"attn_tc_{w.name}.md")
+    traffic, traffic_src = profiled_traffic(f"attn_tc_{w.name}.md")
+    if args.layers is not None:
+        traffic, traffic_src = None, "profiling slice: no summary for this layer count"
     roofline = {"bound": "tensor", "achieved": round(attn_tflops, 2), "peak": pk["bf16_tflops"],
                 "unit": "TFLOP/s", "frac": round(attn_tflops / pk["bf16_tflops"], 4),
-                "traffic": traffic, "kernel": "attn_tc_kernel",
-                "peak_source": pk["source"] + " (burst)"}
+                "traffic": traffic, "traffic_source": traffic_src, "kernel": "attn_tc_kernel",
+                "peak_source": pk["source"] + " (burst)",
+                "frac_of_sustained": (round(attn_tflops / pk["bf16_tflops_sustained"], 4)
+                                      if pk.get("bf16_tflops_sustained") else None),
+                "algorithmic": "FLOP = 4 * 128 * Hq * L * sum(qpos + 1) over the step's selection"}
     if w.dtype == "f32":
         roofline.update({"bound": "alu", "kernel": "attn_f32_kernel", "peak": None, "frac": None})
-    rs_bytes = rb_bytes + sc_bytes
+    rs_bytes = W.rebase_score_bytes(w, fused)
     kernels = {
         "rebase_score": {"us": round(seq[0] * 1e3, 2), "bytes": rs_bytes,
                          "gbs": round(rs_bytes / (seq[0] / 1e3) / 1e9, 1),
                          "frac_hbm": round(rs_bytes / (seq[0] / 1e3) / 1e9 / pk["hbm_gbs"], 4),
                          "launches": 1 if fused else 2,
+                         "bytes_counted": ("re-base r+w of every moved key row; score: fresh rows "
+                                           "read + fp32 written" + (" (the re-based rows are "
+                                           "read back from L2 inside the launch)" if fused else
+                                           " + re-based rows read again")),
                          "timed": f"event around the call, {seq_steps} steps after the timed loop"},
         "select": {"us": round(seq[1] * 1e3, 2), "bytes": sel_bytes,
                    "gbs": round(sel_bytes / (seq[1] / 1e3) / 1e9, 1),
@@ -261,6 +308,22 @@ def run_gpu(args, w, ws, rank, local):
                       "frac_tensor": round(attn_tflops / pk["bf16_tflops"], 4),
                       "timed": "in the timed loop, events on its stream around the call"},
     }
+    config = config_of(w, ws)
+    if args.layers is not None:
+        config["profiling_slice"] = f"first {w.n_layers} layers only (--layers)"
+
+    line = {
+        "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": ws,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 5),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": w.dtype, "data": DATA, "config": config,
+        "roofline": roofline, "kernels": kernels,
+        "gpu_launches": launches_per_step * args.steps,
+        "clocks": clk,
+        "wall_s_timed_loop": round(wall, 4),
+    }
+    if args.no_e2e:
+        return line, x, pristine
 
     # ---- end to end through the public API: host buffers, copies inside the timed region
     host = {"k": pristine.cpu().pin_memory(), "v": x["v"].cpu().pin_memory(),
@@ -306,117 +369,279 @@ def run_gpu(args, w, ws, rank, local):
     e2e_mean = max_over_ranks(pipe_mean, dev)
     graph_mean = max_over_ranks(graph_mean, dev)
     eager_mean = max_over_ranks(eager_mean, dev)
-    line = {
-        "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": ws,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 5),
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": w.dtype,
-        "data": "synthetic: seeded N(0,1) stored keys/values/queries, lognormal fresh-key "
-                "deviation, Qwen2.5-VL-shaped",
-        "config": {"workload": w.name, "layers": w.n_layers, "chunks": w.n_chunks,
-                   "tokens_per_chunk": w.chunk_tokens, "T": w.T, "T_vis": w.t_vis,
-                   "q_heads": w.hq, "kv_heads": w.hkv, "rho": w.rho_bp / 1e4, "k": w.k,
-                   "suffix_rows": w.suffix,
-                   "l2": "flushed between steps (256 MB write) and stored keys restored, untimed",
-                   "parallelism": f"{ws} independent replica(s)"},
-        "roofline": roofline,
-        "kernels": kernels,
-        "e2e": {"value": round(replica_throughput(w.t_vis, e2e_mean, ws), 1), "unit": UNIT,
-                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                "ms_per_step": round(e2e_mean, 4),
-                "ms_min_median_max": pipe_spread,
-                "steps": e2e_steps,
-                "path": "PipelinedQuery.replay (copies and kernels overlapped by layer group, "
-                        "one CUDA graph)",
-                "graph_value": round(replica_throughput(w.t_vis, graph_mean, ws), 1),
-                "eager_value": round(replica_throughput(w.t_vis, eager_mean, ws), 1)},
-        "gpu_launches": launches_per_step * args.steps,
-        "clocks": clk,
-        "wall_s_timed_loop": round(wall, 4),
-    }
-    return line
+    line["e2e"] = {"value": round(replica_throughput(w.t_vis, e2e_mean, ws), 1), "unit": UNIT,
+                   "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                   "ms_per_step": round(e2e_mean, 4),
+                   "ms_min_median_max": pipe_spread,
+                   "steps": e2e_steps,
+                   "h2d_gbs_effective": round(h2d / (e2e_mean / 1e3) / 1e9, 1),
+                   "path": "PipelinedQuery.replay (copies and kernels overlapped by layer "
+                           "group, one CUDA graph)",
+                   "graph_value": round(replica_throughput(w.t_vis, graph_mean, ws), 1),
+                   "eager_value": round(replica_throughput(w.t_vis, eager_mean, ws), 1)}
+    # the CPU-baseline leg reads the GPU arm's own inputs (not its results)
+    return line, x, pristine
 
 
 # ----------------------------------------------------------------------------- oracle
 
-def oracle_step(w, st, layers):
-    """The oracle's composition query restricted to `layers` for re-base and attention
-    (score and select always full).  Returns seconds per phase."""
+# Oracle worker state: the sampled inputs as .npy files in a scratch directory, opened
+# as memory maps by the parent and by every worker process of the pool.
+_ORC = {}
+
+
+def _oracle_init(workdir: str, meta: dict):
+    """Opens the sample's arrays (in the parent for the 1-process run, in each worker)."""
     import oracle as O
-    t = {}
-    loc, glo = st["loc"], st["glo"]
-    cand = slice(w.cand0, w.cand0 + w.n_cand)
-    t0 = time.perf_counter()
-    k_r = {l: O.rebase(st["k"][l][None], loc, glo, w.dtype)[0][0] for l in layers}
-    t["rebase"] = time.perf_counter() - t0
-    t0 = time.perf_counter()
-    kc = O.rebase(st["k_score"][None], loc[cand], glo[cand], w.dtype)[0][0]
-    score = O.score_f32_canonical(st["fresh"].astype(np.float32), kc.astype(np.float32))
-    t["score"] = time.perf_counter() - t0
-    t0 = time.perf_counter()
-    sel = O.select_topk(score, w.k, w.cand0)
-    qpos = np.concatenate([sel, np.arange(w.T - w.suffix, w.T)]).astype(np.int32)
-    t["select"] = time.perf_counter() - t0
-    t0 = time.perf_counter()
-    for l in layers:
-        O.repair_attention(st["q"][l][None], k_r[l][None], st["v"][l][None], qpos)
-    t["attention"] = time.perf_counter() - t0
-    return t
+    _ORC.clear()
+    _ORC.update(meta)
+    _ORC["O"] = O
+    ld = lambda name, mode="r": np.load(os.path.join(workdir, name + ".npy"), mmap_mode=mode)  # noqa: E731
+    for l in meta["layers"]:
+        _ORC[("k", l)] = ld(f"k{l}")
+        _ORC[("v", l)] = ld(f"v{l}")
+        _ORC[("q", l)] = ld(f"q{l}")
+    _ORC["fresh32"] = ld("fresh32")
+    _ORC["loc"] = ld("loc")
+    _ORC["glo"] = ld("glo")
+    _ORC["dir"] = workdir
 
 
-def oracle_state(w, seed, layers):
-    import oracle as O
-    x = W.make_inputs(w, seed=seed, device="cpu")
-    loc, glo = W.coordinates(w)
-    cand = slice(w.cand0, w.cand0 + w.n_cand)
-    f = lambda t: t.float().numpy().astype(np.float64)   # noqa: E731
-    st = {"loc": loc, "glo": glo, "k": {l: f(x["k"][l]) for l in layers},
-          "v": {l: f(x["v"][l]) for l in layers}, "q": {l: f(x["q"][l]) for l in layers},
-          "k_score": f(x["k"][w.score_layer, cand])}
-    st["fresh"] = O.rebase(f(x["k_fresh_local"])[None], loc[cand], glo[cand], w.dtype)[0][0]
-    return st
+def _kr(l, sid):
+    """Re-based keys of layer l for step sid: a new file every step (rewriting pages of a
+    file under writeback would stall the writer)."""
+    key = ("kr", l, sid)
+    if key not in _ORC:
+        for old in [k for k in _ORC if isinstance(k, tuple) and k[0] == "kr"]:
+            del _ORC[old]
+        _ORC[key] = np.load(os.path.join(_ORC["dir"], f"kr{l}_{sid}.npy"), mmap_mode="r+")
+    return _ORC[key]
 
 
-def oracle_rate(w, seed, layers, steps):
-    """Composed visual tokens/s of the oracle, scaling the per-layer phases to all layers."""
-    st = oracle_state(w, seed, layers)
-    times = []
-    for _ in range(steps):
-        t = oracle_step(w, st, layers)
-        scale = w.n_layers / len(layers)
-        times.append(t["score"] + t["select"] + scale * (t["rebase"] + t["attention"]))
-    return w.t_vis / float(np.mean(times)), times
+def _oracle_rebase(task):
+    l, sid, a, b = task
+    O = _ORC["O"]
+    out = O.rebase(np.asarray(_ORC[("k", l)][a:b])[None], _ORC["loc"][a:b], _ORC["glo"][a:b],
+                   _ORC["dtype"])[0][0]
+    _kr(l, sid)[a:b] = out
+    return b - a
 
 
-def cpu_baseline(w, seed, layers, steps):
-    rate, times = oracle_rate(w, seed, layers, steps)
-    return {"value": round(rate, 2), "unit": UNIT, "cores": 1, "kind": "oracle",
-            "sample": f"{steps} step(s); re-base and attention timed on layers {list(layers)} of "
-                      f"{w.n_layers} and scaled by {w.n_layers}/{len(layers)}; score and select "
-                      f"over all {w.n_cand} candidates; numpy, 1 thread",
-            "seconds_per_full_step_est": round(float(np.mean(times)), 3)}
+def _oracle_score(task):
+    sid, a, b = task
+    c0, sl = _ORC["cand0"], _ORC["score_layer"]
+    kc = np.asarray(_kr(sl, sid)[c0 + a:c0 + b]).astype(np.float32)
+    return _ORC["O"].score_f32_canonical(np.asarray(_ORC["fresh32"][a:b]), kc)
 
 
-def run_reference(args, w):
+def _oracle_attention(task):
+    l, sid, rows, qpos = task
+    _ORC["O"].repair_attention(_ORC[("q", l)][None], _kr(l, sid)[None], _ORC[("v", l)][None],
+                               qpos, rows=rows)
+    return len(rows)
+
+
+class OracleSample:
+    """The oracle's composition query on a bounded sample of one workload.
+
+    One sampled step: re-base of the layers in `layers` (all tokens), score and
+    selection over every candidate (on the re-based score layer), and repair
+    attention of a seeded sample of query rows at those layers.  The full step is
+    estimated by scaling the re-base by L / len(layers) and the attention by
+    (L / len(layers)) * sum over all rows of (qpos + 1) / the same sum over the
+    sampled rows (its work is linear in the visible keys).  With a process pool the
+    work is split by token range, candidate range and row subset over worker
+    processes (spawned, so none inherits a CUDA context); the oracle's functions
+    run unchanged on each part.
+    """
+
+    def __init__(self, w, k, v, q, fresh_local, layers):
+        import shutil
+        import tempfile
+
+        import oracle as O
+        self.w = w
+        self.layers = list(layers)
+        if w.score_layer not in self.layers:
+            raise ValueError("the sampled layers must include the score layer")
+        # a memory-backed directory when it has room for the sample, else the temp directory
+        need = 8 * (3 * k[self.layers[0]].size + q[self.layers[0]].size) * len(self.layers)
+        base = None
+        if os.path.isdir("/dev/shm"):
+            try:
+                if shutil.disk_usage("/dev/shm").free > 2 * need:
+                    base = "/dev/shm"
+            except OSError:
+                pass
+        self.dir = tempfile.mkdtemp(prefix="cs_oracle_", dir=base)
+        self.sid = 0
+        loc, glo = W.coordinates(w)
+        cand = slice(w.cand0, w.cand0 + w.n_cand)
+        # set-up, untimed: the fresh keys at global coordinates (the shallow recompute's output)
+        fresh = O.rebase(fresh_local[None], loc[cand], glo[cand], w.dtype)[0][0]
+        sv = lambda name, a: np.save(os.path.join(self.dir, name + ".npy"), a)  # noqa: E731
+        for l in self.layers:
+            sv(f"k{l}", k[l])
+            sv(f"v{l}", v[l])
+            sv(f"q{l}", q[l])
+        self.kshape = k[self.layers[0]].shape
+        sv("fresh32", fresh.astype(np.float32))
+        sv("loc", loc)
+        sv("glo", glo)
+        self.meta = {"layers": self.layers, "dtype": w.dtype, "cand0": w.cand0,
+                     "score_layer": w.score_layer}
+        self.pool = None
+        self.workers = 1
+
+    @classmethod
+    def from_tensors(cls, w, x, layers):
+        """Inputs copied from the tensors of make_inputs (layer i of x = layers[i])."""
+        f = lambda t: t.detach().float().cpu().numpy().astype(np.float64)   # noqa: E731
+        return cls(w, {l: f(x["k"][i]) for i, l in enumerate(layers)},
+                   {l: f(x["v"][i]) for i, l in enumerate(layers)},
+                   {l: f(x["q"][i]) for i, l in enumerate(layers)}, f(x["k_fresh_local"]), layers)
+
+    def start(self, workers: int):
+        """Runs the next steps on `workers` processes (1: in this process)."""
+        import multiprocessing as mp
+        self.stop()
+        self.workers = workers
+        if workers > 1:
+            self.pool = mp.get_context("spawn").Pool(workers, initializer=_oracle_init,
+                                                     initargs=(self.dir, self.meta))
+        _oracle_init(self.dir, self.meta)
+
+    def stop(self):
+        if self.pool is not None:
+            self.pool.close()
+            self.pool.join()
+            self.pool = None
+
+    def close(self):
+        import shutil
+        self.stop()
+        _ORC.clear()
+        shutil.rmtree(self.dir, ignore_errors=True)
+
+    @staticmethod
+    def _split(n, parts):
+        edges = np.linspace(0, n, max(1, min(parts, n)) + 1).astype(int)
+        return [(int(a), int(b)) for a, b in zip(edges[:-1], edges[1:]) if b > a]
+
+    def _map(self, fn, items):
+        if self.pool is None:
+            return [fn(i) for i in items]
+        return self.pool.map(fn, items, chunksize=1)
+
+    def step(self, n_rows: int, row_seed: int):
+        w, p = self.w, self.workers
+        sid = self.sid = self.sid + 1
+        for l in self.layers:   # untimed: this step's output files (the previous step's go)
+            np.lib.format.open_memmap(os.path.join(self.dir, f"kr{l}_{sid}.npy"), mode="w+",
+                                      dtype=np.float64, shape=self.kshape).flush()
+            old = os.path.join(self.dir, f"kr{l}_{sid - 1}.npy")
+            if os.path.exists(old):
+                os.unlink(old)
+        t = {}
+        t0 = time.perf_counter()
+        self._map(_oracle_rebase, [(l, sid, a, b) for l in self.layers
+                                   for a, b in self._split(w.T, p)])
+        t["rebase"] = time.perf_counter() - t0
+        t0 = time.perf_counter()
+        parts = self._map(_oracle_score, [(sid, a, b) for a, b in self._split(w.n_cand, p)])
+        score = np.concatenate(parts) if parts else np.zeros(0, np.float32)
+        t["score"] = time.perf_counter() - t0
+        t0 = time.perf_counter()
+        sel = _ORC["O"].select_topk(score, w.k, w.cand0)
+        qpos = np.concatenate([sel, np.arange(w.T - w.suffix, w.T)]).astype(np.int32)
+        t["select"] = time.perf_counter() - t0
+        rows = W.sample_rows(w.M, n_rows, seed=row_seed)
+        # interleaved row subsets: each worker gets early and late rows alike
+        subsets = [rows[i::p] for i in range(min(p, len(rows)))]
+        t0 = time.perf_counter()
+        self._map(_oracle_attention, [(l, sid, r, qpos) for l in self.layers for r in subsets])
+        t["attention"] = time.perf_counter() - t0
+        lay = w.n_layers / len(self.layers)
+        vis_all = float(np.sum(qpos.astype(np.float64) + 1.0))
+        vis_rows = float(np.sum(qpos[rows].astype(np.float64) + 1.0))
+        attn_scale = lay * vis_all / vis_rows if len(rows) else 0.0
+        t["sampled_s"] = t["rebase"] + t["score"] + t["select"] + t["attention"]
+        t["full_step_s_est"] = (lay * t["rebase"] + t["score"] + t["select"]
+                                + attn_scale * t["attention"])
+        t["rows"] = int(len(rows))
+        t["attn_scale"] = attn_scale
+        return t
+
+    def describe(self, n_rows: int) -> str:
+        w = self.w
+        return (f"re-base of layer(s) {self.layers} of {w.n_layers} (all {w.T} tokens, scaled by "
+                f"{w.n_layers}/{len(self.layers)}); score and select over all {w.n_cand} "
+                f"candidates; attention of {min(n_rows, w.M)} of {w.M} query rows (seeded, first "
+                f"and last included) at those layers, scaled by {w.n_layers}/{len(self.layers)} "
+                f"x sum(qpos+1) over all rows / over the sampled rows; numpy fp64")
+
+    def rate(self, workers: int, steps: int, n_rows: int, seed0: int = 0):
+        """(tokens/s of the estimated full step, per-step timing dicts)."""
+        self.start(workers)
+        try:
+            times = [self.step(n_rows, row_seed=seed0 + s) for s in range(steps)]
+        finally:
+            self.stop()
+        full = float(np.mean([t["full_step_s_est"] for t in times]))
+        return self.w.t_vis / full, times
+
+
+def cpu_baseline(w, x, layers, n_rows):
+    """The oracle on the GPU machine's host, 1 process and all cores, on the GPU arm's own inputs."""
+    sample = OracleSample.from_tensors(w, x, layers)
+    cores = host_cores()
+    try:
+        r1, t1 = sample.rate(1, 1, n_rows)
+        rn, tn = sample.rate(cores, 1, n_rows)
+    finally:
+        sample.close()
+    return {"value": round(rn, 2), "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": "1 step; " + sample.describe(n_rows) + f"; {cores} worker processes",
+            "cpu_model": cpu_model(),
+            "sampled_s": round(tn[0]["sampled_s"], 3),
+            "full_step_s_est": round(tn[0]["full_step_s_est"], 3),
+            "single_thread": {"value": round(r1, 2), "unit": UNIT, "cores": 1,
+                              "sampled_s": round(t1[0]["sampled_s"], 3),
+                              "full_step_s_est": round(t1[0]["full_step_s_est"], 3)}}
+
+
+def run_reference(args, w, ws):
+    """The reference arm: the oracle (the paper publishes no code) on the host cores."""
     layers = [w.score_layer]
-    st = oracle_state(w, args.seed, layers)
-    for _ in range(args.warmup):
-        oracle_step(w, st, layers)
-    times = []
-    for _ in range(max(1, args.steps)):
-        t = oracle_step(w, st, layers)
-        times.append(t["score"] + t["select"] + w.n_layers / len(layers) * (t["rebase"] + t["attention"]))
-    rate = w.t_vis / float(np.mean(times))
-    ms = float(np.mean(times)) * 1e3
-    cb = {"value": round(rate, 2), "unit": UNIT, "cores": 1, "kind": "oracle",
-          "sample": f"each step: re-base and attention of layer {layers} scaled by "
-                    f"{w.n_layers}, score and select over all candidates; numpy, 1 thread"}
+    x = W.make_inputs(w, seed=args.seed, device="cpu", layers=layers)
+    sample = OracleSample.from_tensors(w, x, layers)
+    del x
+    cores = host_cores()
+    try:
+        sample.start(cores)
+        for s in range(args.warmup):
+            sample.step(args.cpu_rows, row_seed=1000 + s)
+        wall0 = time.perf_counter()
+        times = [sample.step(args.cpu_rows, row_seed=s) for s in range(args.steps)]
+        wall = time.perf_counter() - wall0
+    finally:
+        sample.close()
+    full = float(np.mean([t["full_step_s_est"] for t in times]))
+    rate = w.t_vis / full
+    ms_sampled = 1e3 * float(np.mean([t["sampled_s"] for t in times]))
+    desc = (f"each of the {args.steps} timed steps: " + sample.describe(args.cpu_rows)
+            + f" (a new row sample per step); {cores} worker processes")
     return {"impl": "reference", "metric": METRIC, "value": round(rate, 2), "unit": UNIT,
-            "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 3),
+            "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(ms_sampled, 3),
+            "ms_per_step_is": "wall time of one sampled step as run (the timed region is "
+                              "steps x this); value is T_vis / the estimated full-step time",
+            "full_step_ms_est": round(1e3 * full, 3),
+            "wall_s_timed_loop": round(wall, 3),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic, same workload as the GPU arm",
-            "config": {"workload": w.name, "T": w.T, "T_vis": w.t_vis, "k": w.k},
-            "cpu_baseline": cb,
+            "data": DATA + " (CPU generator)", "config": config_of(w, ws),
+            "cpu_baseline": {"value": round(rate, 2), "unit": UNIT, "cores": cores,
+                             "kind": "oracle", "sample": desc, "cpu_model": cpu_model()},
             "e2e": {"value": round(rate, 2), "unit": UNIT, "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
 
@@ -424,8 +649,8 @@ def run_reference(args, w):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=100)
-    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--workload", default=W.BENCH_WORKLOAD, choices=sorted(W.CONFIGS))
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--seed", type=int, default=0)
@@ -433,22 +658,33 @@ def main():
     ap.add_argument("--no-fuse", action="store_true",
                     help="run re-base and score as two calls (the standalone score kernel), "
                          "not the fused cs_rebase_and_score launch")
-    ap.add_argument("--cpu-layers", type=int, default=2)
+    ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end (host buffer) leg")
+    ap.add_argument("--layers", type=int, default=None,
+                    help="profiling aid: run only the first N layers of the workload (the line "
+                         "says so; not a headline number)")
+    ap.add_argument("--cpu-rows", type=int, default=256,
+                    help="query rows the oracle attends per sampled step")
     args = ap.parse_args()
     w = W.CONFIGS[args.workload]
+    if args.layers is not None:
+        if not 1 <= args.layers <= w.n_layers:
+            ap.error("--layers must be in [1, n_layers]")
+        w = w.with_(n_layers=args.layers)
     ws, rank, local = _dist_env()
 
     if args.impl == "reference":
         if rank == 0:
-            print(json.dumps(run_reference(args, w)), flush=True)
+            print(json.dumps(run_reference(args, w, ws)), flush=True)
         return
 
     if ws > 1:
         torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local))
-    line = run_gpu(args, w, ws, rank, local)
+    line, x, pristine = run_gpu(args, w, ws, rank, local)
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
-        layers = list(range(min(args.cpu_layers, w.n_layers)))
-        line["cpu_baseline"] = cpu_baseline(w, args.seed, layers, steps=1)
+        layers = [w.score_layer]
+        xs = {"k": pristine[layers], "v": x["v"][layers], "q": x["q"][layers],
+              "k_fresh_local": x["k_fresh_local"]}
+        line["cpu_baseline"] = cpu_baseline(w, xs, layers, args.cpu_rows)
     if rank == 0:
         print(json.dumps(line), flush=True)
     if ws > 1:

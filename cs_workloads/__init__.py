@@ -139,8 +139,9 @@ CONFIGS = {
                                dtype="bf16"),
 }
 
-# The workload the throughput number is quoted on (3B shape, 4 chunks x 1024 tokens).
-BENCH_WORKLOAD = "qwen3b_4x1024"
+# The workload the throughput number is quoted on: the largest single-GPU configuration
+# of the 3B shape (64 chunks x 1024 tokens, the middle of its rho sweep).
+BENCH_WORKLOAD = "qwen3b_64x1024_r15"
 
 
 def coordinates(w: Workload):
@@ -186,8 +187,10 @@ def coordinates(w: Workload):
     return loc.astype(np.int32), glo.astype(np.int32)
 
 
-def seed_for(w: Workload, seed: int, tensor_id: int) -> int:
-    return (seed * 1000003 + sum(map(ord, w.name)) * 101 + tensor_id) & 0x7FFFFFFF
+def seed_for(w: Workload, seed: int, tensor_id: int, layer: int = 0) -> int:
+    """Seed of one drawn tensor (and, for per-layer tensors, of one of its layers)."""
+    base = seed * 1000003 + sum(map(ord, w.name)) * 101 + tensor_id
+    return (base * 1009 + layer) & 0x7FFFFFFF
 
 
 def _randn(shape, seed, device):
@@ -196,7 +199,16 @@ def _randn(shape, seed, device):
     return torch.randn(shape, generator=g, device=device, dtype=torch.float32)
 
 
-def make_inputs(w: Workload, seed: int = 0, device="cpu"):
+def _per_layer(w: Workload, shape, seed: int, tensor_id: int, layers, device, dtype):
+    """[len(layers), *shape] in `dtype`; layer l is drawn from its own seed, so any
+    subset of layers can be materialised without drawing the others."""
+    out = torch.empty((len(layers),) + tuple(shape), dtype=dtype, device=device)
+    for i, l in enumerate(layers):
+        out[i] = _randn(shape, seed_for(w, seed, tensor_id, l), device).to(dtype)
+    return out
+
+
+def make_inputs(w: Workload, seed: int = 0, device="cpu", layers=None):
     """Seeded synthetic inputs for one composition query.
 
     Returns a dict of tensors on `device`:
@@ -204,18 +216,25 @@ def make_inputs(w: Workload, seed: int = 0, device="cpu"):
       q [L,M,Hq,D]                   queries of the repaired rows (storage dtype)
       k_fresh_local [Nc,Hkv,D]       perturbed layer-1 stored keys, local coords
       pos_local, pos_global [T,3]    int32 coordinates
-    The draws use torch's generator for `device`; the same (workload, seed,
-    device) always gives the same tensors.
+    Every layer of k, v and q is drawn from its own seed.  `layers` (a list of layer
+    indices) materialises only those layers, in that order (the leading dimension is
+    then len(layers)); k_fresh_local is the same whichever layers are asked for.  The
+    draws use torch's generator for `device`; the same (workload, seed, device)
+    always gives the same tensors.
     """
-    L, T, Hkv, Hq, D = w.n_layers, w.T, w.hkv, w.hq, w.head_dim
+    T, Hkv, Hq, D = w.T, w.hkv, w.hq, w.head_dim
     dt = w.torch_dtype
-    k = _randn((L, T, Hkv, D), seed_for(w, seed, 1), device).to(dt)
-    v = _randn((L, T, Hkv, D), seed_for(w, seed, 2), device).to(dt)
-    q = _randn((L, w.M, Hq, D), seed_for(w, seed, 3), device).to(dt)
+    layers = list(range(w.n_layers)) if layers is None else [int(l) for l in layers]
+    k = _per_layer(w, (T, Hkv, D), seed, 1, layers, device, dt)
+    v = _per_layer(w, (T, Hkv, D), seed, 2, layers, device, dt)
+    q = _per_layer(w, (w.M, Hq, D), seed, 3, layers, device, dt)
     nc = w.n_cand
     scale = torch.exp(w.sigma * _randn((nc, 1, 1), seed_for(w, seed, 4), device))
     eps = _randn((nc, Hkv, D), seed_for(w, seed, 5), device)
-    base = k[w.score_layer, w.cand0:w.cand0 + nc].float()
+    sl = w.score_layer
+    k_sl = k[layers.index(sl)] if sl in layers else _per_layer(w, (T, Hkv, D), seed, 1, [sl],
+                                                               device, dt)[0]
+    base = k_sl[w.cand0:w.cand0 + nc].float()
     k_fresh_local = (base + scale * eps).to(dt)
     loc, glo = coordinates(w)
     return {
@@ -260,10 +279,18 @@ def score_bytes(w: Workload) -> float:
     return w.n_cand * (2.0 * w.hkv * w.head_dim * w.elem_bytes + 4.0)
 
 
+def rebase_score_bytes(w: Workload, fused: bool) -> float:
+    """Algorithmic bytes of re-base + score.  Fused into one launch, the score reads the
+    fresh rows and writes one fp32 per candidate from HBM, and reads the rows it has just
+    re-based back from L2 (not counted); as two launches it also reads those rows again."""
+    fresh = w.n_cand * (w.hkv * w.head_dim * w.elem_bytes + 4.0)
+    return rebase_bytes(w) + (fresh if fused else score_bytes(w))
+
+
 def k_from_rho(rho_bp: int, n_cand: int) -> int:
     return (rho_bp * n_cand + 9999) // 10000
 
 
 __all__ = ["Workload", "CONFIGS", "BENCH_WORKLOAD", "coordinates", "make_inputs",
            "random_coordinates", "sample_rows", "attention_flops", "rebase_bytes",
-           "score_bytes", "k_from_rho", "HEAD_DIM", "MROPE_SECTIONS", "ROPE_THETA"]
+           "score_bytes", "rebase_score_bytes", "k_from_rho", "HEAD_DIM", "MROPE_SECTIONS", "ROPE_THETA"]

@@ -18,15 +18,18 @@
  *     default stream).  Argument checks run on the host before any launch; a
  *     call that returns an error launched nothing.
  *   - Data-dependent failures found on the device (a bounded wait that gave
- *     up, a query position out of range) are recorded in a per-device status
- *     word and reported by cs_sync_status().
+ *     up, a query position out of range) are recorded in a status word that
+ *     is shared by every stream of the device (and every caller of this
+ *     library in the process), and reported by cs_sync_status().
  *   - There is no CPU fallback: every computation runs in this library's own
  *     CUDA kernels.
  *   - head_dim must be 128 (CS_ERR_UNSUPPORTED otherwise).  Every tensor
  *     pointer and every row start must be 16-byte aligned.
  *   - The library owns no device allocation.  Its one piece of device state
- *     is a small static status word per device, set up on the first call
- *     made on that device; make that first call before capturing a stream.
+ *     is a small static status word per device, whose address is looked up on
+ *     the first call made on that device (and again after the device's
+ *     context changes, e.g. after cudaDeviceReset); make that first call
+ *     before capturing a stream.
  */
 #ifndef CHRONOSTITCH_H
 #define CHRONOSTITCH_H
@@ -170,7 +173,8 @@ cs_status cs_select_topk(const float *score, int n, int k, int32_t idx_base, int
  *            device; a violation yields CS_ERR_DEVICE_ARG at cs_sync_status and
  *            leaves o undefined)
  *   lse      optional fp32 [n_layers][M][n_q_heads]: the natural-log normaliser
- *            log(sum_j exp(scale * q.k_j)); NULL to skip
+ *            log(sum_j exp(scale * q.k_j)); NULL to skip; 4-byte aligned and
+ *            not overlapping k, v or o (CS_ERR_INVALID_ARG)
  *   scale    the logit scale, 1/sqrt(head_dim) in Eq. 1
  * bf16 runs on the tensor cores (bf16 operands, fp32 accumulation); f32 runs
  * fp32 arithmetic on the CUDA cores.
@@ -203,9 +207,17 @@ cs_status cs_scatter_rows(void *cache, const void *rows, cs_dtype dtype, int n_l
                           int row_elems, const int32_t *idx, void *stream);
 
 /*
- * Waits for `stream`, then reports and clears the device status word of the
- * current device: CS_ERR_TIMEOUT or CS_ERR_DEVICE_ARG if a kernel recorded one
- * since the last call, CS_ERR_CUDA if the stream reported an error, else CS_OK.
+ * Takes the device status record of the current device and waits for `stream`:
+ * CS_ERR_TIMEOUT or CS_ERR_DEVICE_ARG if a kernel recorded an error since the
+ * last take, CS_ERR_CUDA if the stream reported an error, else CS_OK.
+ *
+ * The record is device-wide: it holds the first error recorded by any kernel
+ * of this library on the device, on any stream, until it is taken.  The take
+ * runs on the device in `stream`'s order (one atomic exchange with zero), so
+ * it covers every kernel issued earlier on `stream`; an error recorded
+ * concurrently by a kernel on another stream is either taken by this call
+ * (and reported here, against this stream) or left for the next call, never
+ * lost.  Calls from several host threads are serialised.
  */
 cs_status cs_sync_status(void *stream);
 

@@ -105,6 +105,18 @@ def _stream(stream):
     return int(stream)
 
 
+def _fresh(stream, make):
+    """An output tensor allocated here for a call launched on `stream`.  torch's caching
+    allocator tracks the current stream; when the call runs on another one, the tensor is
+    recorded on it, so its memory is not handed out again before the kernel has written it."""
+    t = make()
+    if stream is not None:
+        s = stream if isinstance(stream, torch.cuda.Stream) else torch.cuda.ExternalStream(int(stream))
+        if s.cuda_stream != torch.cuda.current_stream(t.device).cuda_stream:
+            t.record_stream(s)
+    return t
+
+
 def _dtype_code(t: torch.Tensor) -> int:
     if t.dtype == torch.bfloat16:
         return CS_DTYPE_BF16
@@ -186,7 +198,7 @@ def cs_rebase_and_score(k: torch.Tensor, pos_local: torch.Tensor, pos_global: to
     _inner_contiguous(k_fresh, "k_fresh")
     n = k_fresh.shape[0]
     if score_out is None:
-        score_out = torch.empty(n, dtype=torch.float32, device=k.device)
+        score_out = _fresh(stream, lambda: torch.empty(n, dtype=torch.float32, device=k.device))
     _need_cuda(score_out)
     if score_out.dtype != torch.float32 or score_out.numel() < n or not score_out.is_contiguous():
         raise ValueError("score_out must be contiguous fp32 with n elements")
@@ -211,7 +223,7 @@ def cs_score_deviation(k_fresh: torch.Tensor, k_cached: torch.Tensor, *,
     _inner_contiguous(k_cached, "k_cached")
     n, H, D = k_fresh.shape
     if out is None:
-        out = torch.empty(n, dtype=torch.float32, device=k_fresh.device)
+        out = _fresh(stream, lambda: torch.empty(n, dtype=torch.float32, device=k_fresh.device))
     _need_cuda(out)
     if out.dtype != torch.float32 or out.numel() < n or not out.is_contiguous():
         raise ValueError("out must be contiguous fp32 with n elements")
@@ -230,7 +242,7 @@ def cs_select_topk(score: torch.Tensor, k: int, idx_base: int = 0, *,
     if score.dtype != torch.float32 or score.dim() != 1 or not score.is_contiguous():
         raise ValueError("score must be contiguous fp32 [n]")
     if out is None:
-        out = torch.empty(int(k), dtype=torch.int32, device=score.device)
+        out = _fresh(stream, lambda: torch.empty(int(k), dtype=torch.int32, device=score.device))
     _need_cuda(out)
     if out.dtype != torch.int32 or out.numel() < k or not out.is_contiguous():
         raise ValueError("out must be contiguous int32 with k elements")
@@ -257,7 +269,7 @@ def cs_repair_attention(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, qpos:
     if qpos.dtype != torch.int32 or qpos.numel() != M or not qpos.is_contiguous():
         raise ValueError("qpos must be contiguous int32 [M]")
     if out is None:
-        out = torch.empty_like(q)
+        out = _fresh(stream, lambda: torch.empty_like(q))
     _need_cuda(out)
     if out.shape != q.shape or out.dtype != q.dtype or not out.is_contiguous():
         raise ValueError("out must match q")

@@ -1,6 +1,8 @@
 // C ABI entry points of libchronostitch: argument validation on the host,
 // kernel launches, and the per-device status word that kernels write when
 // they detect a data error or a bounded wait gives up.
+#include <cuda.h>
+
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -12,8 +14,8 @@
 
 namespace cs {
 
-// Per-device status word (static storage of this module, one copy per device).
-__device__ unsigned int g_status[kStatusWords];
+// Per-device status area (static storage of this module, one copy per device).
+__device__ __align__(16) unsigned int g_status[kStatusWords];
 
 namespace {
 
@@ -22,6 +24,33 @@ thread_local char t_detail[512] = "no error";
 constexpr int kMaxDevices = 64;
 std::mutex g_mu;
 unsigned int *g_status_addr[kMaxDevices] = {};
+CUcontext g_status_ctx[kMaxDevices] = {};
+std::mutex g_take_mu;   // one take at a time: the take slot (words 2-3) is shared
+
+using CtxGetCurrentFn = CUresult (*)(CUcontext *);
+
+// The driver's cuCtxGetCurrent, through the runtime's entry-point query (no link
+// against the driver library); nullptr if unavailable.
+CtxGetCurrentFn ctx_get_current_fn() {
+    static CtxGetCurrentFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *ptr = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &ptr, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<CtxGetCurrentFn>(ptr);
+    });
+    return fn;
+}
+
+CUcontext current_ctx() {
+    CUcontext c = nullptr;
+    CtxGetCurrentFn fn = ctx_get_current_fn();
+    if (fn == nullptr || fn(&c) != CUDA_SUCCESS) return nullptr;
+    return c;
+}
 
 cudaStream_t as_stream(void *s) { return static_cast<cudaStream_t>(s); }
 
@@ -67,8 +96,11 @@ unsigned int *status_word() {
         fail(CS_ERR_UNSUPPORTED, "device ordinal %d beyond %d", dev, kMaxDevices);
         return nullptr;
     }
+    // the address belongs to the context the module was loaded in: after a device reset
+    // (a new primary context) it is looked up again
+    const CUcontext ctx = current_ctx();
     std::lock_guard<std::mutex> lock(g_mu);
-    if (g_status_addr[dev] == nullptr) {
+    if (g_status_addr[dev] == nullptr || ctx == nullptr || g_status_ctx[dev] != ctx) {
         void *p = nullptr;
         e = cudaGetSymbolAddress(&p, g_status);
         if (e != cudaSuccess) {
@@ -76,8 +108,16 @@ unsigned int *status_word() {
             return nullptr;
         }
         g_status_addr[dev] = static_cast<unsigned int *>(p);
+        g_status_ctx[dev] = current_ctx();   // the look-up may have created the context
     }
     return g_status_addr[dev];
+}
+
+int sm_count() {
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+    return n;
 }
 
 }  // namespace cs
@@ -339,6 +379,8 @@ cs_status cs_repair_attention(const void *q, const void *k, const void *v, void 
     if (n_q_heads / n_kv_heads > 128)
         return fail(CS_ERR_UNSUPPORTED, "more than 128 query heads per kv head");
     if (!std::isfinite(scale)) return fail(CS_ERR_INVALID_ARG, "scale must be finite");
+    if (lse != nullptr && (reinterpret_cast<uintptr_t>(lse) & 3u))
+        return fail(CS_ERR_INVALID_ARG, "lse must be 4-byte aligned");
     if (kv_layer_stride < static_cast<long long>(T) * n_kv_heads * head_dim)
         return fail(CS_ERR_INVALID_ARG, "kv_layer_stride < T*n_kv_heads*head_dim");
     if (n_layers == 0 || M == 0) return CS_OK;
@@ -362,6 +404,15 @@ cs_status cs_repair_attention(const void *q, const void *k, const void *v, void 
         const char *vc = static_cast<const char *>(v);
         if ((oc < kc + kv_span && kc < oc + o_span) || (oc < vc + kv_span && vc < oc + o_span))
             return fail(CS_ERR_INVALID_ARG, "o overlaps k or v");
+        // lse is written while other CTAs still read k and v, too
+        if (lse != nullptr) {
+            const long long l_span = 4ll * n_layers * M * n_q_heads;
+            const char *lc = reinterpret_cast<const char *>(lse);
+            if ((lc < kc + kv_span && kc < lc + l_span) || (lc < vc + kv_span && vc < lc + l_span))
+                return fail(CS_ERR_INVALID_ARG, "lse overlaps k or v");
+            if (lc < oc + o_span && oc < lc + l_span)
+                return fail(CS_ERR_INVALID_ARG, "lse overlaps o");
+        }
     }
     unsigned int *status = status_word();
     if (status == nullptr) return CS_ERR_CUDA;
@@ -389,19 +440,28 @@ cs_status cs_repair_attention(const void *q, const void *k, const void *v, void 
 }
 
 cs_status cs_sync_status(void *stream) {
-    cudaError_t e = cudaStreamSynchronize(as_stream(stream));
-    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
     unsigned int *status = status_word();
     if (status == nullptr) return CS_ERR_CUDA;
-    unsigned int host[kStatusWords] = {0, 0, 0, 0};
-    e = cudaMemcpy(host, status, sizeof(host), cudaMemcpyDeviceToHost);
-    if (e != cudaSuccess) return cuda_fail(e, "reading the status word");
-    if (host[0] == 0) return CS_OK;
-    const unsigned int zero[kStatusWords] = {0, 0, 0, 0};
-    e = cudaMemcpy(status, zero, sizeof(zero), cudaMemcpyHostToDevice);
-    if (e != cudaSuccess) return cuda_fail(e, "clearing the status word");
-    const cs_status s = host[0] == 4u ? CS_ERR_TIMEOUT : CS_ERR_DEVICE_ARG;
-    return fail(s, "device status %u at site %u (detail %u)", host[0], host[1], host[2]);
+    const cudaStream_t s = as_stream(stream);
+    unsigned long long rec = 0;
+    {
+        // take the record on the device, in `stream`'s order (exchange with 0, so an error
+        // recorded concurrently by a kernel on another stream is either taken now or left
+        // for the next call), then wait for the stream and read what was taken
+        std::lock_guard<std::mutex> lock(g_take_mu);
+        cudaError_t e = launch_status_take(status, s);
+        if (e != cudaSuccess) return cuda_fail(e, "status take launch");
+        e = cudaMemcpyAsync(&rec, status + 2, sizeof(rec), cudaMemcpyDeviceToHost, s);
+        if (e != cudaSuccess) return cuda_fail(e, "reading the status record");
+        e = cudaStreamSynchronize(s);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+    }
+    if (rec == 0) return CS_OK;
+    const unsigned int code = static_cast<unsigned int>(rec >> 56);
+    const unsigned int site = static_cast<unsigned int>((rec >> 48) & 0xFFu);
+    const unsigned int detail = static_cast<unsigned int>(rec & 0xFFFFFFFFu);
+    const cs_status st = code == 4u ? CS_ERR_TIMEOUT : CS_ERR_DEVICE_ARG;
+    return fail(st, "device status %u at site %u (detail %u)", code, site, detail);
 }
 
 }  // extern "C"
@@ -425,6 +485,20 @@ __global__ void wait_timeout_kernel(unsigned int *status, unsigned long long lim
 
 cudaError_t launch_wait_timeout(unsigned int *status, unsigned int limit_us, cudaStream_t s) {
     wait_timeout_kernel<<<1, 1, 0, s>>>(status, 1000ull * limit_us);
+    return cudaGetLastError();
+}
+
+namespace {
+// Moves the status record (words 0-1) into the take slot (words 2-3) and clears it,
+// in one atomic exchange.
+__global__ void status_take_kernel(unsigned int *status) {
+    unsigned long long *w = reinterpret_cast<unsigned long long *>(status);
+    w[1] = atomicExch(&w[0], 0ull);
+}
+}  // namespace
+
+cudaError_t launch_status_take(unsigned int *status, cudaStream_t s) {
+    status_take_kernel<<<1, 1, 0, s>>>(status);
     return cudaGetLastError();
 }
 }  // namespace cs

@@ -9,7 +9,7 @@
 
 namespace cs {
 
-// Site tags stored in status word[1].
+// Site tags of a status record.
 enum : unsigned int {
     kSiteAttnProducer = 1,
     kSiteAttnMma = 2,
@@ -19,14 +19,17 @@ enum : unsigned int {
     kSiteScatter = 6,
 };
 
-// Records the first error on this device: word[0] = code, word[1] = site, word[2] = detail.
+// Records the first error on this device.  The record is one 64-bit word (the first
+// two 32-bit words of the status area, 8-byte aligned): code in bits 56-63, site in
+// bits 48-55, detail in bits 0-31; 0 means no error.  A compare-and-swap from 0 keeps
+// the first error, and the host's take (an exchange with 0, cs_sync_status) removes a
+// whole record at once, so no record is torn or lost.
 __device__ __forceinline__ void report_error(unsigned int *status, unsigned int code,
                                              unsigned int site, unsigned int detail) {
     if (status == nullptr) return;
-    if (atomicCAS(status, 0u, code) == 0u) {
-        status[1] = site;
-        status[2] = detail;
-    }
+    const unsigned long long rec = (static_cast<unsigned long long>(code & 0xFFu) << 56) |
+                                   (static_cast<unsigned long long>(site & 0xFFu) << 48) | detail;
+    atomicCAS(reinterpret_cast<unsigned long long *>(status), 0ull, rec);
 }
 
 // ---------------------------------------------------------------------------

@@ -8,15 +8,19 @@
 
 namespace cs {
 
-// Device status word layout (one per device, zeroed by cs_sync_status):
-//   word[0]  first error code recorded (CS_ERR_TIMEOUT / CS_ERR_DEVICE_ARG), 0 if none
-//   word[1]  where it happened (kernel-specific site tag)
-//   word[2]  extra detail (block index, row, ...)
+// Device status area (one per device, 16-byte aligned, four 32-bit words):
+//   words 0-1  the first error recorded since the last take, as one 64-bit record
+//              (code << 56 | site << 48 | detail; see report_error), 0 if none
+//   words 2-3  where cs_sync_status's take kernel leaves the record it removed
 constexpr int kStatusWords = 4;
 
-// Returns the device address of the status word of the current device, or
+// Returns the device address of the status area of the current device (looked up
+// again whenever the current CUDA context differs from the one it was found in), or
 // nullptr on a CUDA error (the detail is recorded for cs_last_error_detail).
 unsigned int *status_word();
+
+// Number of SMs of the current device (0 if it cannot be queried).
+int sm_count();
 
 // Records a detail string for cs_last_error_detail and returns `s`.
 cs_status fail(cs_status s, const char *fmt, ...);
@@ -105,5 +109,7 @@ cudaError_t launch_attn_f32(const AttnArgs &a, cudaStream_t s);
 cs_status launch_attn_tc(const AttnArgs &a, cudaStream_t s);
 
 cudaError_t launch_wait_timeout(unsigned int *status, unsigned int limit_us, cudaStream_t s);
+// Takes the status record into the take slot and clears it (cs_sync_status).
+cudaError_t launch_status_take(unsigned int *status, cudaStream_t s);
 
 }  // namespace cs

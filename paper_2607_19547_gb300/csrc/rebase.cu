@@ -486,7 +486,8 @@ cudaError_t launch_rebase(const RebaseArgs &a, cs_dtype dt, cudaStream_t s) {
         // split layers across CTAs only when there are too few token blocks to fill
         // the GPU (every extra CTA repeats the cos/sin prologue)
         int groups = 1;
-        const int target = 152 * 2;
+        const int sms = sm_count();
+        const int target = (sms > 0 ? sms : 152) * 2;
         if (blocks < target) groups = std::min((target + blocks - 1) / blocks,
                                                (a.n_layers + slots - 1) / slots);
         const int l_per_cta = (a.n_layers + groups - 1) / groups;

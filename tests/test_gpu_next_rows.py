@@ -94,6 +94,40 @@ def test_naive_policy_keeps_stored_keys(cslib):
     assert np.array_equal(bits16(x["k"]), before)
 
 
+@pytest.mark.parametrize("name", ["tiny_f32", "qwen3b_4x1024"])
+def test_naive_policy_end_to_end_matches_oracle(cslib, name):
+    """Table 1's naive concatenation: the stored keys stay at their chunk-local positions.
+    Score, selection and the attention of sampled rows equal the oracle's on the un-rebased
+    cache, with the fresh keys at global coordinates as the recompute would give them."""
+    w = W.CONFIGS[name]
+    x = W.make_inputs(w, seed=8, device="cuda")
+    loc, glo = W.coordinates(w)
+    cand = slice(w.cand0, w.cand0 + w.n_cand)
+    layers = [0, w.n_layers - 1] if w.n_layers > 1 else [0]
+    stored_k = {l: f64(x["k"][l]) for l in layers}
+    k_score = f64(x["k"][w.score_layer, cand])
+    fresh_local = f64(x["k_fresh_local"])
+    fresh = torch.empty_like(x["k_fresh_local"])
+    cslib.cs_rebase_keys(x["k_fresh_local"][None], cuda(loc[cand]), cuda(glo[cand]),
+                         k_out=fresh[None])
+    q = ComposedQuery(_shape(w), w.torch_dtype)
+    out, qpos = q.step(x["k"], x["v"], x["q"], fresh, cuda(loc), cuda(glo), policy="naive")
+    cslib.cs_sync_status()
+    # the oracle: its own fresh keys at global coordinates, the stored keys as they are
+    kf, _ = O.rebase(fresh_local[None], loc[cand], glo[cand], w.dtype)
+    score = O.score_f32_canonical(kf[0].astype(np.float32), k_score.astype(np.float32))
+    assert np.array_equal(q.score.cpu().numpy().view(np.uint32), score.view(np.uint32))
+    sel = O.select_topk(score, w.k, w.cand0)
+    exp_qpos = np.concatenate([sel, np.arange(w.T - w.suffix, w.T)]).astype(np.int32)
+    assert np.array_equal(qpos.cpu().numpy(), exp_qpos)
+    rows = W.sample_rows(w.M, 32, seed=10)
+    for l in layers:
+        eo, _ = O.repair_attention(f64(x["q"][l])[None][:, rows], stored_k[l][None],
+                                   f64(x["v"][l])[None], exp_qpos[rows])
+        go = f64(out[l][torch.as_tensor(rows, device="cuda")])[None]
+        assert np.max(np.abs(go - eo)) <= TOL[w.dtype]
+
+
 def test_pipeline_with_scatter_back_matches_oracle(cslib):
     """Fresh K/V of the repaired rows go into the cache before the attention: the attention of
     sampled rows equals the oracle's over the oracle-composed cache with those rows replaced."""

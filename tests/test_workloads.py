@@ -68,3 +68,15 @@ def test_sample_rows_keeps_ends():
     r = W.sample_rows(1000, 50, seed=1)
     assert r[0] == 0 and r[-1] == 999 and len(r) == 50 and np.all(np.diff(r) > 0)
     assert list(W.sample_rows(5, 50, seed=1)) == [0, 1, 2, 3, 4]
+
+
+def test_layer_subset_matches_full_draw():
+    """Every layer has its own seed: a subset of layers is the same tensors as the full draw,
+    and the fresh keys do not depend on which layers were asked for."""
+    w = W.CONFIGS["qwen3b_4x1024"].with_(n_layers=3, n_chunks=2, grid_t=1, grid_h=4, grid_w=4)
+    full = W.make_inputs(w, seed=5)
+    sub = W.make_inputs(w, seed=5, layers=[2, 0])
+    for key in ("k", "v", "q"):
+        assert torch.equal(sub[key][0], full[key][2]) and torch.equal(sub[key][1], full[key][0])
+    assert torch.equal(sub["k_fresh_local"], full["k_fresh_local"])
+    assert not torch.equal(full["k"][0], full["k"][1])
