@@ -204,52 +204,45 @@ __device__ bool build_table(const RebaseArgs &a, int t0, int TB, int (*s_delta)[
 // Each output r ~ u c - w s is evaluated in fp32 with
 //   |r - exact| <= 2.5 * 2^-24 * (|x| + |y|) + 2^-149
 // (c_hi and s_hi lie within 2^-25 of cos and sin; one rounding of the product,
-// one of the fma; the last term covers subnormal results), so
-// E = 3 * 2^-24 * fl(|x| + |y|) + 2^-148, rounded once, exceeds the error
-// strictly.  The bf16 rounding of r is certain when
-//   (1) the midpoint m of r's own bf16 interval (|r| truncated to bf16 plus half
-//       a bf16 unit: an fp32 number in r's binade, so |r| - m is exact) lies at
-//       least E away from |r|, and
-//   (2) |r| >= 1024 E: for |r| in [2^e, 2^(e+1)) this makes E < 2^(e-9), the
-//       least distance from r to any other midpoint (the one just below a power
-//       of two included; subnormal r alike, with midpoints 2^-134 apart).
-// Each condition is a difference that rounds to a negative number exactly when
-// it fails, so the sign bits of all 32 differences are OR-ed and tested once.
-// Non-finite and huge inputs (where r could overflow) fail through the sum of
-// |x| + |y| over the slice, which must compare below 2^126 (NaN compares false).
+// one of the fma; the last term covers subnormal results).  With
+//   E = fl(4 * 2^-24 * fl(|x| + |y|) + 2^-147),
+// lo = fl(r - E) and hi = fl(r + E) bracket the exact value: E exceeds the error
+// bound by 1.5 * 2^-24 (|x| + |y|) + 2^-148, more than the rounding error of either
+// sum (at most 2^-24 (|r| + E), or 2^-150 for subnormal sums).  Rounding to nearest
+// (ties to even) is monotone, so when lo and hi round to the same bf16 value the
+// exact value rounds to it too, and so does r (lo <= r <= hi).  The test is
+// therefore: round lo and hi of two adjacent outputs with one packed conversion
+// each and compare the two words.  A non-finite input or an overflowing sum makes
+// lo and hi differ (an infinity meets a NaN or the other infinity), except a NaN
+// input, whose NaN output is accepted as it is.
 __device__ __forceinline__ bool rotate_slice(const uint4 &xv, const uint4 &yv, const float (&c)[8],
                                              const float (&sn)[8], uint32_t (&ow)[4],
                                              uint32_t (&pw)[4]) {
     const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w};
     const uint32_t yw[4] = {yv.x, yv.y, yv.z, yv.w};
-    uint32_t neg = 0;
-    float usum = 0.0f;
+    const float2 kE = make_float2(0x1p-22f, 0x1p-22f);       // 4 * 2^-24
+    const float2 kT = make_float2(0x1p-147f, 0x1p-147f);
+    const float2 kM = make_float2(-1.0f, -1.0f);
+    uint32_t diff = 0;
 #pragma unroll
     for (int w = 0; w < 4; ++w) {
-        float r1[2], r2[2];
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-            const int e = 2 * w + h;
-            const float x = h ? bf16_hi(xw[w]) : bf16_lo(xw[w]);
-            const float y = h ? bf16_hi(yw[w]) : bf16_lo(yw[w]);
-            r1[h] = __fmaf_rn(x, c[e], -__fmul_rn(y, sn[e]));    // x c - y s
-            r2[h] = __fmaf_rn(y, c[e], __fmul_rn(x, sn[e]));     // y c + x s
-            const float u = __fadd_rn(fabsf(x), fabsf(y));
-            usum = __fadd_rn(usum, u);
-            const float E = __fmaf_rn(u, 0x1.8p-23f, 0x1p-148f);
-            const float E2 = __fmul_rn(E, 1024.0f);
-            const float a1 = fabsf(r1[h]), a2 = fabsf(r2[h]);
-            const float m1 = __uint_as_float((__float_as_uint(r1[h]) & 0x7FFF0000u) | 0x8000u);
-            const float m2 = __uint_as_float((__float_as_uint(r2[h]) & 0x7FFF0000u) | 0x8000u);
-            neg |= __float_as_uint(__fsub_rn(fabsf(__fsub_rn(a1, m1)), E)) |
-                   __float_as_uint(__fsub_rn(a1, E2));
-            neg |= __float_as_uint(__fsub_rn(fabsf(__fsub_rn(a2, m2)), E)) |
-                   __float_as_uint(__fsub_rn(a2, E2));
-        }
-        ow[w] = pack_bf16x2_rn(r1[0], r1[1]);
-        pw[w] = pack_bf16x2_rn(r2[0], r2[1]);
+        const int e0 = 2 * w, e1 = 2 * w + 1;
+        const float x0 = bf16_lo(xw[w]), x1 = bf16_hi(xw[w]);
+        const float y0 = bf16_lo(yw[w]), y1 = bf16_hi(yw[w]);
+        const float2 r1 = make_float2(__fmaf_rn(x0, c[e0], -__fmul_rn(y0, sn[e0])),    // x c - y s
+                                      __fmaf_rn(x1, c[e1], -__fmul_rn(y1, sn[e1])));
+        const float2 r2 = make_float2(__fmaf_rn(y0, c[e0], __fmul_rn(x0, sn[e0])),     // y c + x s
+                                      __fmaf_rn(y1, c[e1], __fmul_rn(x1, sn[e1])));
+        const float2 u = make_float2(__fadd_rn(fabsf(x0), fabsf(y0)), __fadd_rn(fabsf(x1), fabsf(y1)));
+        const float2 E = __ffma2_rn(u, kE, kT);
+        const float2 lo1 = __ffma2_rn(E, kM, r1), hi1 = __fadd2_rn(r1, E);
+        const float2 lo2 = __ffma2_rn(E, kM, r2), hi2 = __fadd2_rn(r2, E);
+        diff |= pack_bf16x2_rn(lo1.x, lo1.y) ^ pack_bf16x2_rn(hi1.x, hi1.y);
+        diff |= pack_bf16x2_rn(lo2.x, lo2.y) ^ pack_bf16x2_rn(hi2.x, hi2.y);
+        ow[w] = pack_bf16x2_rn(r1.x, r1.y);
+        pw[w] = pack_bf16x2_rn(r2.x, r2.y);
     }
-    return (neg >> 31) == 0 && usum < 0x1p126f;
+    return diff == 0;
 }
 
 // Eq. 5 block term of the canonical fp32 order: ((q0+q1)+(q2+q3))+((q4+q5)+(q6+q7)),
@@ -296,7 +289,7 @@ __device__ __forceinline__ void stream_slices(const __nv_bfloat16 *src, __nv_bfl
         sn[e] = full[e].z;
     }
     int queued = 0;   // the same on every lane of `part`
-#pragma unroll 2
+#pragma unroll 1
     for (int i = 0; i < count; ++i) {
         if (queued > kQueue - 32) {   // make room for one failing slice per lane
             redo_queue(queued, part, obase, lstep, trow, tab, dst);

@@ -1,27 +1,43 @@
 // Step 3 of the composition path: top-rho selection (ChronoStitch Sec. 2).
 //
-// One CTA of 1024 threads (the candidate scores are a few hundred KB at most and
-// stay in L2).  Scores map to order-preserving 32-bit keys.  Thread t owns the
-// contiguous candidate range [t*per, (t+1)*per); up to 16 keys per thread stay
-// in registers, larger inputs are re-read from L2 in every pass (the histogram
-// passes read them interleaved and coalesced, eight loads in flight).  Up to three
-// MSB-first radix passes over 11-, 11- and 10-bit digits (one shared 2048-bin
-// histogram, shared-memory atomic increments) find K*, the k-th largest key, and how
-// many keys equal to K* belong to the top k (the lowest-index ones: the
-// tie-break); they stop early once every key left in K*'s bin is taken, and the
-// resolved prefix of K* then stands for it.  One block-wide scan of the per-thread (greater, equal) counts
-// then gives every selected index its output position, so the output is
-// ascending without a sort.
+// Scores map to order-preserving 32-bit keys; the k largest keys win, equal keys
+// rank the lower index first, and the output is the selected indices in
+// ascending order.  Exact radix select over one thread-block cluster of C CTAs
+// (C = 1, 2, 4, 8 or 16, sized from n):
+//   - CTA r owns the contiguous candidate range [r*span, (r+1)*span) and thread t
+//     of it the contiguous range [t*per, (t+1)*per) inside that; up to 16 keys per
+//     thread stay in registers (16-byte loads), larger inputs are re-read in every
+//     pass;
+//   - up to three MSB-first passes over 11-, 11- and 10-bit digits find K*, the
+//     k-th largest key, and how many keys equal to K* are taken (the lowest-index
+//     ones).  A pass: every CTA counts its own keys that match the digits resolved
+//     so far into a 2048-bin histogram in its shared memory; after a cluster
+//     barrier CTA r sums bin slice r (2048/C bins) over all C histograms through
+//     distributed shared memory; after a second barrier every CTA reads the C
+//     slice totals and the one slice that holds the k-th key and takes the same
+//     decision.  The histogram is double-buffered by pass parity, so a CTA never
+//     clears a buffer that another CTA may still read.  The passes stop once every
+//     key left in K*'s bin is taken;
+//   - one block-wide scan of the per-thread (greater, equal) counts, plus the
+//     counts of the CTAs before it (read from their shared memory), gives every
+//     thread its first output position, so the output is ascending without a sort.
+// The cluster barriers are hardware barriers that every thread of every CTA
+// reaches the same number of times (the decisions are identical in every CTA); a
+// final barrier keeps each CTA's shared memory alive until the others have read it.
+// No global memory besides the scores and the output is used.
+#include <algorithm>
+#include <mutex>
+
 #include "cs_device.cuh"
 #include "cs_internal.h"
 
 namespace cs {
 namespace {
 
-constexpr int kThreads = 1024;
-constexpr int kWarps = kThreads / 32;
+constexpr int kNT = 512;          // threads per CTA
+constexpr int kWarps = kNT / 32;
 constexpr int kBins = 2048;
-constexpr int kRegKeys = 16;   // keys per thread held in registers (n <= 16384)
+constexpr int kMaxCluster = 16;
 
 // Order-preserving key of an fp32 bit pattern u (scores are read as raw 32-bit
 // words, never as floats, so every NaN payload and sign survives).
@@ -29,15 +45,42 @@ __device__ __forceinline__ uint32_t order_key(uint32_t u) {
     return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
-// hist[d] += 1 for every lane with `active`.  Plain shared-memory atomics: lanes
-// that share a digit (scores of one binade often do) were measured faster this way
-// than aggregated with __match_any_sync first (10.7 / 18.3 / 59.7 us against 12.6 /
-// 29.0 / 112 us for 3 072 / 15 360 / 64 512 candidates).
-__device__ __forceinline__ void hist_add(uint32_t *hist, uint32_t d, bool active) {
-    if (active) atomicAdd(&hist[d], 1u);
+__device__ __forceinline__ uint32_t cluster_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
 }
 
-// Block-wide inclusive scan of v (all 1024 threads call; wsum holds 32 words).
+// Cluster-wide barrier: release (this CTA's shared-memory writes) / acquire.
+__device__ __forceinline__ void cluster_arrive() {
+    asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() {
+    asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_sync() {
+    cluster_arrive();
+    cluster_wait();
+}
+
+// Address of `p` (this CTA's shared memory) in the shared memory of CTA `rank`.
+__device__ __forceinline__ uint32_t dsmem_addr(const void *p, uint32_t rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_u32(p)), "r"(rank));
+    return r;
+}
+__device__ __forceinline__ uint32_t dsmem_ld(uint32_t addr) {
+    uint32_t v;
+    asm volatile("ld.shared::cluster.u32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
+    return v;
+}
+__device__ __forceinline__ unsigned long long dsmem_ld64(uint32_t addr) {
+    unsigned long long v;
+    asm volatile("ld.shared::cluster.u64 %0, [%1];" : "=l"(v) : "r"(addr) : "memory");
+    return v;
+}
+
+// Block-wide inclusive scan of v (all kNT threads call; wsum holds kWarps words).
 // Callers separate two uses of wsum with a barrier.
 template <typename T>
 __device__ __forceinline__ T block_incl_scan(T v, T *wsum) {
@@ -50,154 +93,339 @@ __device__ __forceinline__ T block_incl_scan(T v, T *wsum) {
     if (lane == 31) wsum[warp] = v;
     __syncthreads();
     if (warp == 0) {
-        T w = wsum[lane];
+        T w = lane < kWarps ? wsum[lane] : T(0);
 #pragma unroll
-        for (int o = 1; o < 32; o *= 2) {
+        for (int o = 1; o < kWarps; o *= 2) {
             const T y = __shfl_up_sync(0xFFFFFFFFu, w, o);
             if (lane >= o) w += y;
         }
-        wsum[lane] = w;
+        if (lane < kWarps) wsum[lane] = w;
     }
     __syncthreads();
     return warp > 0 ? v + wsum[warp - 1] : v;
 }
 
-// KPT > 0: exactly KPT keys per thread in registers; KPT == 0: per keys per
-// thread read from global memory in every pass.
+struct SelShared {
+    uint32_t hist[2][kBins];            // per-pass histograms (double-buffered)
+    uint32_t red[kBins];                // this CTA's reduced bin slice (C > 1)
+    uint32_t part[kNT];                 // partial sums of the slice reduction
+    uint32_t wtot[kWarps];              // per-warp sums of the slice total
+    unsigned long long wsum[kWarps];    // block scan scratch
+    unsigned long long cta_counts;      // this CTA's (greater << 32 | equal) in the final phase
+    uint32_t slice_total;               // sum of red[]
+    uint32_t s_digit, s_krem, s_done;   // the pass's decision
+    uint32_t s_hit, s_above, s_cnt;     // bin search result inside the block
+    unsigned long long s_before;        // counts of the CTAs before this one
+};
+
+// Finds, among S bin counts read through get(j) (j = 0..S-1, ascending digits), the
+// bin that holds the krem-th largest key: sets s->s_hit = that bin, s->s_above = the
+// keys in higher bins and s->s_cnt = the keys in that bin.  Every thread calls it (it
+// contains block barriers).
+template <typename Get>
+__device__ __forceinline__ void find_bin(SelShared *s, int S, uint32_t krem, Get get) {
+    const int t = threadIdx.x;
+    if (t == 0) {   // defined results even if no bin were found (the counts rule it out)
+        s->s_hit = 0;
+        s->s_above = 0;
+        s->s_cnt = 0;
+    }
+    const int q = (S + kNT - 1) / kNT;     // bins per thread, walked from the top
+    const int hi = S - t * q;              // thread t: bins [hi - q, hi) (clipped at 0)
+    uint32_t v[4] = {0, 0, 0, 0};          // q <= 4 (S <= 2048)
+    uint32_t mine = 0;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int j = hi - 1 - i;
+        if (i < q && j >= 0) v[i] = get(j);
+        mine += v[i];
+    }
+    const unsigned long long incl = block_incl_scan<unsigned long long>(mine, s->wsum);
+    const unsigned long long above = incl - mine;
+    if (above < krem && incl >= krem) {
+        unsigned long long acc = above;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            if (i < q && acc + v[i] >= krem) {
+                s->s_hit = static_cast<uint32_t>(hi - 1 - i);
+                s->s_above = static_cast<uint32_t>(acc);
+                s->s_cnt = v[i];
+                break;
+            }
+            acc += v[i];
+        }
+    }
+    __syncthreads();
+}
+
+// KPT > 0: exactly KPT keys per thread in registers (per == KPT); KPT == 0: `per`
+// keys per thread (a multiple of 4) re-read from global memory in every pass.
+// vec: the scores start 16-byte aligned (16-byte loads where a group of 4 is whole).
 template <int KPT>
-__global__ void __launch_bounds__(kThreads, 1)
-select_kernel(const uint32_t *__restrict__ score, int n, int k, int idx_base, int per,
+__global__ void __launch_bounds__(kNT, 1)
+select_kernel(const uint32_t *__restrict__ score, int n, int k, int idx_base, int per, int vec,
               int *__restrict__ out) {
     pdl_wait();   // inputs may come from the previous kernel of the stream
     pdl_trigger();
-    __shared__ uint32_t hist[kBins];
-    __shared__ unsigned long long wsum[kWarps];
-    __shared__ uint32_t s_digit, s_krem, s_done;
-    const int tid = threadIdx.x;
+    __shared__ __align__(16) SelShared sh;
+    SelShared *s = &sh;
+    const int t = threadIdx.x;
+    const uint32_t C = gridDim.x;                // one cluster spans the grid
+    const uint32_t r = C > 1 ? cluster_rank() : 0u;
+    const long long i0 = (static_cast<long long>(r) * kNT + t) * per;   // first key of this thread
+    const int cnt = static_cast<int>(max(0ll, min(static_cast<long long>(per), n - i0)));
 
-    if (k >= n) {   // everything is selected, in index order
-        for (int i = tid; i < n; i += kThreads) out[i] = idx_base + i;
+    if (k >= n) {   // everything is selected, in index order (no barrier on this path)
+        for (int i = 0; i < cnt; ++i) out[i0 + i] = idx_base + static_cast<int>(i0) + i;
         return;
     }
-    const int i0 = tid * per;
-    const int cnt = max(0, min(per, n - i0));
-    uint32_t reg[KPT > 0 ? KPT : 1];
+
+    // keys of this thread, four at a time
+    auto load4 = [&](int c, uint32_t (&kb)[4]) {
+        const long long g = i0 + 4 * c;
+        if (vec && 4 * c + 3 < cnt) {
+            const uint4 u = __ldg(reinterpret_cast<const uint4 *>(score + g));
+            kb[0] = order_key(u.x); kb[1] = order_key(u.y);
+            kb[2] = order_key(u.z); kb[3] = order_key(u.w);
+        } else {
+#pragma unroll
+            for (int e = 0; e < 4; ++e) kb[e] = 4 * c + e < cnt ? order_key(__ldg(score + g + e)) : 0u;
+        }
+    };
+    constexpr int kRegs = KPT > 0 ? KPT : 4;
+    uint32_t reg[kRegs];
     if (KPT > 0) {
 #pragma unroll
-        for (int i = 0; i < (KPT > 0 ? KPT : 1); ++i)
-            reg[i] = i < cnt ? order_key(__ldg(score + i0 + i)) : 0u;
+        for (int c = 0; c < kRegs / 4; ++c) {
+            uint32_t kb[4];
+            load4(c, kb);
+#pragma unroll
+            for (int e = 0; e < 4; ++e) reg[4 * c + e] = kb[e];
+        }
     }
-    auto key_at = [&](int i) -> uint32_t {
-        if (KPT > 0) return reg[i];
-        return order_key(__ldg(score + i0 + i));
+    // calls f(local index, key) for every key of this thread, in index order
+    auto for_keys = [&](auto f) {
+        if (KPT > 0) {
+#pragma unroll
+            for (int i = 0; i < kRegs; ++i)
+                if (i < cnt) f(i, reg[i]);
+        } else {
+            for (int c = 0; 4 * c < cnt; ++c) {
+                uint32_t kb[4];
+                load4(c, kb);
+#pragma unroll
+                for (int e = 0; e < 4; ++e)
+                    if (4 * c + e < cnt) f(4 * c + e, kb[e]);
+            }
+        }
     };
 
+    for (int j = t; j < 2 * kBins; j += kNT) (&s->hist[0][0])[j] = 0u;
+    __syncthreads();
+
+    const int S = kBins / static_cast<int>(C);   // bins of one slice
     uint32_t prefix = 0, pmask = 0, krem = static_cast<uint32_t>(k);
 #pragma unroll 1
     for (int pass = 0; pass < 3; ++pass) {
         const int shift = pass == 0 ? 21 : (pass == 1 ? 10 : 0);
         const uint32_t dmask = pass == 2 ? 0x3FFu : 0x7FFu;
-        for (int b = tid; b < kBins; b += kThreads) hist[b] = 0;
-        __syncthreads();
-        if (KPT > 0) {
-#pragma unroll
-            for (int i = 0; i < (KPT > 0 ? KPT : 1); ++i) {
-                const uint32_t key = reg[i];
-                hist_add(hist, (key >> shift) & dmask, i < cnt && (key & pmask) == prefix);
-            }
+        uint32_t *hist = s->hist[pass & 1];
+        for_keys([&](int, uint32_t key) {
+            if ((key & pmask) == prefix) atomicAdd(&hist[(key >> shift) & dmask], 1u);
+        });
+        uint32_t digit, above;
+        if (C == 1) {
+            __syncthreads();
+            find_bin(s, kBins, krem, [&](int j) { return hist[j]; });
+            digit = s->s_hit;
+            above = s->s_above;
+            // the other buffer is cleared for the next pass (nobody else reads it)
+            for (int j = t; j < kBins; j += kNT) s->hist[(pass + 1) & 1][j] = 0u;
         } else {
-            // the histogram does not care which thread counts which key: read the keys
-            // interleaved (coalesced), eight loads in flight before their increments
-            const int rounds = (n + kThreads * 8 - 1) / (kThreads * 8);   // uniform
-            for (int rr = 0; rr < rounds; ++rr) {
-                uint32_t kb[8];
-#pragma unroll
-                for (int u = 0; u < 8; ++u) {
-                    const int i = (rr * 8 + u) * kThreads + tid;
-                    kb[u] = i < n ? order_key(__ldg(score + i)) : 0u;
+            cluster_sync();
+            // every CTA has finished reading the other buffer (last pass): clear it
+            for (int j = t; j < kBins; j += kNT) s->hist[(pass + 1) & 1][j] = 0u;
+            // reduce bin slice r over the C histograms of the cluster
+            uint32_t tot = 0;
+            if (S >= kNT) {
+                for (int bl = t; bl < S; bl += kNT) {
+                    uint32_t v = 0;
+                    for (uint32_t src = 0; src < C; ++src)
+                        v += dsmem_ld(dsmem_addr(&hist[r * S + bl], src));
+                    s->red[bl] = v;
+                    tot += v;
                 }
-#pragma unroll
-                for (int u = 0; u < 8; ++u) {
-                    const int i = (rr * 8 + u) * kThreads + tid;
-                    hist_add(hist, (kb[u] >> shift) & dmask, i < n && (kb[u] & pmask) == prefix);
-                }
-            }
-        }
-        __syncthreads();
-        // thread t holds bins 2047-2t and 2046-2t; an inclusive scan from the top
-        // finds the bin in which the k-th largest key falls
-        const uint32_t hi = hist[kBins - 1 - 2 * tid], lo = hist[kBins - 2 - 2 * tid];
-        const unsigned long long incl =
-            block_incl_scan<unsigned long long>(static_cast<unsigned long long>(hi + lo), wsum);
-        const unsigned long long above = incl - (hi + lo);
-        if (above < krem && incl >= krem) {
-            // the bin holding the k-th largest key; when every key left in it is taken,
-            // the remaining digits cannot change the selection and the passes stop
-            if (above + hi >= krem) {
-                s_digit = static_cast<uint32_t>(kBins - 1 - 2 * tid);
-                s_krem = krem - static_cast<uint32_t>(above);
-                s_done = hi == s_krem;
             } else {
-                s_digit = static_cast<uint32_t>(kBins - 2 - 2 * tid);
-                s_krem = krem - static_cast<uint32_t>(above) - hi;
-                s_done = lo == s_krem;
+                const int G = kNT / S, per_src = static_cast<int>(C) / G;
+                const int bl = t % S, g = t / S;
+                uint32_t v = 0;
+                for (int m = 0; m < per_src; ++m)
+                    v += dsmem_ld(dsmem_addr(&hist[r * S + bl], static_cast<uint32_t>(g * per_src + m)));
+                s->part[t] = v;
+                __syncthreads();
+                if (t < S) {
+                    uint32_t w = 0;
+                    for (int gg = 0; gg < G; ++gg) w += s->part[t + gg * S];
+                    s->red[t] = w;
+                    tot = w;
+                }
             }
+            // slice total
+#pragma unroll
+            for (int o = 16; o >= 1; o /= 2) tot += __shfl_xor_sync(0xFFFFFFFFu, tot, o);
+            if ((t & 31) == 0) s->wtot[t >> 5] = tot;
+            __syncthreads();
+            if (t == 0) {
+                uint32_t a = 0;
+                for (int w = 0; w < kWarps; ++w) a += s->wtot[w];
+                s->slice_total = a;
+            }
+            cluster_sync();
+            // the slice holding the k-th key: slices of higher rank hold higher digits
+            if (t == 0) {
+                s->s_digit = 0;
+                s->s_above = 0;
+            }
+            __syncthreads();
+            if (t < 32) {
+                const uint32_t tj = static_cast<uint32_t>(t) < C
+                                        ? dsmem_ld(dsmem_addr(&s->slice_total, static_cast<uint32_t>(t)))
+                                        : 0u;
+                // inclusive sum over slices >= t (from the top)
+                uint32_t incl = tj;
+#pragma unroll
+                for (int o = 1; o < 32; o *= 2) {
+                    const uint32_t y = __shfl_down_sync(0xFFFFFFFFu, incl, o);
+                    if (t + o < 32) incl += y;
+                }
+                const uint32_t abv = incl - tj;
+                if (static_cast<uint32_t>(t) < C && abv < krem && incl >= krem) {
+                    s->s_digit = static_cast<uint32_t>(t);   // the slice
+                    s->s_above = abv;
+                }
+            }
+            __syncthreads();
+            // (the counts guarantee a slice is found; the clamp keeps every remote
+            // address inside the cluster regardless)
+            const uint32_t sl = min(s->s_digit, C - 1u), above_sl = s->s_above;
+            __syncthreads();   // s_above is rewritten by find_bin
+            find_bin(s, S, krem - above_sl,
+                     [&](int j) { return dsmem_ld(dsmem_addr(&s->red[j], sl)); });
+            digit = sl * static_cast<uint32_t>(S) + s->s_hit;
+            above = above_sl + s->s_above;
         }
-        __syncthreads();
-        prefix |= s_digit << shift;
+        // digit holds the k-th largest key among those with the resolved prefix; when
+        // every key left in its bin is taken the remaining digits cannot change the
+        // selection
+        const uint32_t krem_new = krem - above;
+        const bool done = s->s_cnt == krem_new;
+        prefix |= digit << shift;
         pmask |= dmask << shift;
-        krem = s_krem;
-        if (s_done) break;   // uniform; nothing shared is written again before it is read
-        __syncthreads();     // s_digit / wsum are rewritten by the next pass
+        krem = krem_new;
+        __syncthreads();   // s_hit / s_above / s_digit are rewritten in the next pass
+        if (done) break;   // uniform across the cluster: every CTA took the same decision
     }
-    // prefix = the resolved high bits of K* (all of K* after three passes) and pmask
-    // their mask; krem = how many keys with that prefix are selected (lowest indices first;
-    // all of them when the passes stopped early)
+
+    // prefix = the resolved high bits of K* (all of K* after three passes), pmask their
+    // mask; krem = how many keys with that prefix are selected (lowest indices first)
     const uint32_t kstar = prefix;
     uint32_t gt = 0, eq = 0;
-    if (KPT > 0) {
-#pragma unroll
-        for (int i = 0; i < (KPT > 0 ? KPT : 1); ++i) {
-            gt += (i < cnt && (reg[i] & pmask) > kstar);
-            eq += (i < cnt && (reg[i] & pmask) == kstar);
-        }
-    } else {
-        for (int c0 = 0; c0 < cnt; c0 += 8) {   // eight loads in flight
-            uint32_t kb[8];
-#pragma unroll
-            for (int u = 0; u < 8; ++u) kb[u] = c0 + u < cnt ? (key_at(c0 + u) & pmask) : 0u;
-#pragma unroll
-            for (int u = 0; u < 8; ++u) {
-                gt += c0 + u < cnt && kb[u] > kstar;
-                eq += c0 + u < cnt && kb[u] == kstar;
-            }
-        }
-    }
+    for_keys([&](int, uint32_t key) {
+        gt += (key & pmask) > kstar;
+        eq += (key & pmask) == kstar;
+    });
     const unsigned long long mine = (static_cast<unsigned long long>(gt) << 32) | eq;
-    const unsigned long long before = block_incl_scan<unsigned long long>(mine, wsum) - mine;
+    const unsigned long long incl = block_incl_scan<unsigned long long>(mine, s->wsum);
+    const unsigned long long before_t = incl - mine;
+    if (t == kNT - 1) s->cta_counts = incl;
+    unsigned long long before_cta = 0;
+    if (C > 1) {
+        cluster_sync();
+        if (t < 32) {
+            unsigned long long v = static_cast<uint32_t>(t) < r
+                                       ? dsmem_ld64(dsmem_addr(&s->cta_counts, static_cast<uint32_t>(t)))
+                                       : 0ull;
+#pragma unroll
+            for (int o = 16; o >= 1; o /= 2) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
+            if (t == 0) s->s_before = v;
+        }
+        __syncthreads();
+        before_cta = s->s_before;
+        cluster_arrive();   // this CTA reads no other CTA's shared memory after this point
+    }
+    const unsigned long long before = before_cta + before_t;
     const uint32_t gt_before = static_cast<uint32_t>(before >> 32);
     uint32_t eq_seen = static_cast<uint32_t>(before & 0xFFFFFFFFu);
     uint32_t pos = gt_before + min(eq_seen, krem);
-    if (KPT > 0) {
-#pragma unroll
-        for (int i = 0; i < (KPT > 0 ? KPT : 1); ++i) {
-            const uint32_t key = reg[i] & pmask;
-            if (i < cnt && (key > kstar || (key == kstar && eq_seen++ < krem)))
-                out[pos++] = idx_base + i0 + i;
-        }
-    } else {
-        for (int c0 = 0; c0 < cnt; c0 += 8) {
-            uint32_t kb[8];
-#pragma unroll
-            for (int u = 0; u < 8; ++u) kb[u] = c0 + u < cnt ? (key_at(c0 + u) & pmask) : 0u;
-#pragma unroll
-            for (int u = 0; u < 8; ++u) {
-                const uint32_t key = kb[u];
-                if (c0 + u < cnt && (key > kstar || (key == kstar && eq_seen++ < krem)))
-                    out[pos++] = idx_base + i0 + c0 + u;
+    for_keys([&](int i, uint32_t key) {
+        const uint32_t km = key & pmask;
+        if (km > kstar || (km == kstar && eq_seen++ < krem))
+            out[pos++] = idx_base + static_cast<int>(i0) + i;
+    });
+    if (C > 1) cluster_wait();   // others may still read this CTA's counts until here
+}
+
+// The largest cluster size (a power of two <= 16) the device can co-schedule for
+// kernel number `which` (0..3); cached per kernel and device.
+int max_cluster(int which, void (*kernel)(const uint32_t *, int, int, int, int, int, int *)) {
+    static std::mutex mu;
+    static int cached[4][64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 1;
+    std::lock_guard<std::mutex> lock(mu);
+    int &slot = cached[which][dev];
+    if (slot == 0) {
+        int best = 1;
+        if (cudaFuncSetAttribute(kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+            cudaSuccess)
+            (void)cudaGetLastError();
+        for (int c = kMaxCluster; c >= 2; c /= 2) {
+            cudaLaunchConfig_t cfg = {};
+            cfg.gridDim = dim3(c);
+            cfg.blockDim = dim3(kNT);
+            cudaLaunchAttribute attr[1];
+            attr[0].id = cudaLaunchAttributeClusterDimension;
+            attr[0].val.clusterDim.x = c;
+            attr[0].val.clusterDim.y = 1;
+            attr[0].val.clusterDim.z = 1;
+            cfg.attrs = attr;
+            cfg.numAttrs = 1;
+            int nclusters = 0;
+            if (cudaOccupancyMaxActiveClusters(&nclusters, kernel, &cfg) == cudaSuccess &&
+                nclusters >= 1) {
+                best = c;
+                break;
             }
+            (void)cudaGetLastError();
         }
+        slot = best;
     }
+    return slot;
+}
+
+template <int KPT>
+cudaError_t launch_kpt(int C, const uint32_t *keys, int n, int k, int idx_base, int per, int vec,
+                       int *out, cudaStream_t s) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(C);
+    cfg.blockDim = dim3(kNT);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[2];
+    int na = 0;
+    attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[na].val.programmaticStreamSerializationAllowed = 1;
+    ++na;
+    if (C > 1) {
+        attr[na].id = cudaLaunchAttributeClusterDimension;
+        attr[na].val.clusterDim.x = C;
+        attr[na].val.clusterDim.y = 1;
+        attr[na].val.clusterDim.z = 1;
+        ++na;
+    }
+    cfg.attrs = attr;
+    cfg.numAttrs = na;
+    return cudaLaunchKernelEx(&cfg, select_kernel<KPT>, keys, n, k, idx_base, per, vec, out);
 }
 
 }  // namespace
@@ -206,16 +434,23 @@ cudaError_t launch_select(const float *score, int n, int k, int idx_base, int *o
                           cudaStream_t s) {
     if (k == 0 || n == 0) return cudaSuccess;
     const uint32_t *keys = reinterpret_cast<const uint32_t *>(score);
-    const int per = (n + kThreads - 1) / kThreads;
-    if (per <= 4) {
-        return launch_pdl(select_kernel<4>, dim3(1), dim3(kThreads), 0, s, keys, n, k, idx_base, 4, out);
-    } else if (per <= kRegKeys) {
-        return launch_pdl(select_kernel<kRegKeys>, dim3(1), dim3(kThreads), 0, s, keys, n, k, idx_base,
-                          kRegKeys, out);
-    } else {
-        return launch_pdl(select_kernel<0>, dim3(1), dim3(kThreads), 0, s, keys, n, k, idx_base, per, out);
-    }
-    return cudaGetLastError();
+    const int vec = (reinterpret_cast<uintptr_t>(score) & 15u) == 0;
+    // cluster size: about 4096 keys per CTA, a power of two up to what the device allows
+    int want = 1;
+    while (want < kMaxCluster && static_cast<long long>(want) * 4096 < n) want *= 2;
+    // every variant must be able to run the cluster (the choice of variant below depends on C)
+    int cap = max_cluster(0, select_kernel<4>);
+    cap = std::min(cap, max_cluster(1, select_kernel<8>));
+    cap = std::min(cap, max_cluster(2, select_kernel<16>));
+    cap = std::min(cap, max_cluster(3, select_kernel<0>));
+    const int C = std::min(want, cap);
+    // keys per thread for that cluster: in registers up to 16, else re-read per pass
+    const long long per_thread = (n + static_cast<long long>(C) * kNT - 1) / (static_cast<long long>(C) * kNT);
+    if (per_thread <= 4) return launch_kpt<4>(C, keys, n, k, idx_base, 4, vec, out, s);
+    if (per_thread <= 8) return launch_kpt<8>(C, keys, n, k, idx_base, 8, vec, out, s);
+    if (per_thread <= 16) return launch_kpt<16>(C, keys, n, k, idx_base, 16, vec, out, s);
+    const int per = static_cast<int>((per_thread + 3) / 4 * 4);
+    return launch_kpt<0>(C, keys, n, k, idx_base, per, vec, out, s);
 }
 
 }  // namespace cs

@@ -61,7 +61,10 @@ def _check_select(cs, vals, k, base):
     assert np.array_equal(got.cpu().numpy(), exp)
 
 
-@pytest.mark.parametrize("n", [1, 7, 1023, 1024, 1025, 3072, 4096, 4097, 15360, 16384, 16385, 64512, 100003])
+# n spans every cluster size of the select (1, 2, 4, 8, 16 CTAs), the keys-in-registers
+# variants (4, 8, 16 per thread) and the re-read variant (n > 131072), with ragged tails
+@pytest.mark.parametrize("n", [1, 7, 1023, 1024, 1025, 3072, 4096, 4097, 8191, 8193, 15360, 16384,
+                               16385, 32769, 64512, 100003, 131073, 262147])
 def test_select_matches_oracle(cslib, n):
     rng = np.random.default_rng(n)
     cont = (rng.lognormal(0, 1.5, n) * 256).astype(np.float32)
@@ -93,3 +96,27 @@ def test_select_fraction_of_candidates(cslib):
     assert np.all(np.diff(got) > 0)
     kth = np.sort(vals)[::-1][k - 1]
     assert np.all(vals[got - cand0] >= kth)
+
+
+@pytest.mark.parametrize("n", [5000, 70001])
+def test_select_unaligned_scores(cslib, n):
+    """Scores that start 4 bytes past a 16-byte boundary take the scalar-load path."""
+    rng = np.random.default_rng(n + 1)
+    vals = (rng.lognormal(0, 1.5, n + 1) * 256).astype(np.float32)
+    buf = cuda(vals)
+    view = buf[1:]
+    assert view.data_ptr() % 16 == 4
+    for k in (1, n // 3, n - 1):
+        got = cslib.cs_select_topk(view, k, 9).cpu().numpy()
+        cslib.cs_sync_status()
+        assert np.array_equal(got, O.select_topk(vals[1:], k, 9))
+
+
+def test_select_ties_across_ctas(cslib):
+    """All scores equal over 64 512 candidates (16 CTAs): the k lowest indices, so every
+    CTA's share of the ties depends on the CTAs before it."""
+    n = 64512
+    vals = np.full(n, 7.25, np.float32)
+    vals[::1000] = 9.0
+    for k in (1, 65, 30000, n - 3):
+        _check_select(cslib, vals, k, 1032)
