@@ -125,8 +125,8 @@ cs_status cs_score_deviation(const void *k_fresh, const void *k_cached, cs_dtype
  *                      dtype, n_cand, n_kv_heads, head_dim, fresh_row_stride, E,
  *                      score_out)              with E = n_kv_heads*head_dim,
  * bit for bit, where the candidates are tokens [cand0, cand0 + n_cand) of the
- * cache.  For bf16 with n_kv_heads 1, 2 or 4 it is one kernel launch: the
- * re-base computes the scores of the rows it has just re-based; otherwise two.
+ * cache.  It is one kernel launch: the re-base computes the scores of the rows it
+ * has just re-based (for bf16 and fp32, any supported kv head count).
  *
  *   0 <= score_layer < n_layers (when n_cand > 0);  0 <= cand0,  cand0 + n_cand <= T
  *   k_fresh    row c (token cand0 + c) at k_fresh + c*fresh_row_stride, E elements,

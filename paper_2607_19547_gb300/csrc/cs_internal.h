@@ -65,7 +65,7 @@ struct RebaseArgs {
     unsigned long long turn_step[64];   // theta_i / (2 pi) in units of 2^-64 turns
     unsigned char axis[64];             // sigma(i)
     int in_place;
-    // fused score of layer score_layer (bf16, n_kv_heads 1, 2 or 4): when score_out
+    // fused score of layer score_layer (every supported head count): when score_out
     // is set, score_out[t - cand0] = Eq. 5 squared of fresh row t - cand0 against
     // the re-based row t, for t in [cand0, cand0 + n_cand)
     const void *fresh;

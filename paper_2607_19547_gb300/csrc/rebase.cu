@@ -27,6 +27,7 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kMaxTokensPerCta = 32;   // fp32 kernel
 constexpr int kMaxTokensBf16 = 8;      // bf16 kernel: token block of 8 / n_kv_heads
+constexpr int kMaxBlocks = 512;        // 8-element blocks of one token row (32 kv heads)
 
 // 1/n! split exactly into fp32 hi + lo (hi = fp32(1/n!), lo = fp32(1/n! - hi)).
 __device__ __forceinline__ f2 cf(float hi, float lo) { return {hi, lo}; }
@@ -262,6 +263,33 @@ __device__ __forceinline__ float score_block8(uint4 fv, uint4 cv) {
                      __fadd_rn(__fadd_rn(q[4], q[5]), __fadd_rn(q[6], q[7])));
 }
 
+// Eq. 5's fixed halving order over one token's block sums s[0..B) in shared memory,
+// by one warp: the sums are padded with +0 to a power of two P >= 32 (x + 0 = x for the
+// non-negative block sums, so padding past the canonical power of two changes
+// nothing), lane l holds s[l + 32 j], strides >= 32 are folded in-lane and strides 16
+// .. 1 by an xor butterfly (s[b] + s[b ^ m] = s[b] + s[b + m] for b < m).  Returns the
+// score in every lane.
+__device__ __forceinline__ float reduce_blocks_warp(const float *blk, int B) {
+    constexpr int kMaxJ = kMaxBlocks / 32;
+    const int lane = threadIdx.x & 31;
+    int P = 32;
+    while (P < B) P *= 2;
+    float v[kMaxJ];
+#pragma unroll
+    for (int j = 0; j < kMaxJ; ++j) v[j] = (32 * j < P && lane + 32 * j < B) ? blk[lane + 32 * j] : 0.0f;
+#pragma unroll
+    for (int m = kMaxJ / 2; m >= 1; m /= 2) {
+        if (32 * m < P) {
+#pragma unroll
+            for (int j = 0; j < m; ++j) v[j] = __fadd_rn(v[j], v[j + m]);
+        }
+    }
+    float r = v[0];
+#pragma unroll
+    for (int m = 16; m >= 1; m /= 2) r = __fadd_rn(r, __shfl_xor_sync(0xFFFFFFFFu, r, m));
+    return r;
+}
+
 // The streaming part of the bf16 kernel for one thread's slices (see the kernel
 // below).  `part` holds the lanes of this warp that rotate (moved tokens with
 // layers to walk); they all walk the same number of layers.
@@ -392,6 +420,35 @@ __global__ void __launch_bounds__(kThreads, 4) rebase_bf16_kernel(RebaseArgs a, 
     const unsigned part = __ballot_sync(0xFFFFFFFFu, count > 0 && moved && moved_any);
     if (count > 0)
         stream_slices(src, dst, obase, lstep, count, moved, part, tb * 64 + pg * 8, tab, xv, yv);
+    if (HKV == 0) {
+        // any head count: a token's row may span several warps, so its block sums meet in
+        // shared memory and one warp per token reduces them in the canonical order
+        const bool cta_scores = a.score_out != nullptr && a.score_layer >= l0 &&
+                                a.score_layer < l1 && t0 < a.cand0 + a.n_cand &&
+                                t0 + TB > a.cand0;
+        if (!cta_scores) return;   // the same in every thread of the CTA
+        __shared__ float s_blk[kMaxBlocks];
+        const int B = 16 * hkv;    // blocks of one token row (TB * B <= kMaxBlocks)
+        if (scoring) {
+            const long long o = static_cast<long long>(a.score_layer) * a.layer_stride + row0;
+            const uint4 cx = *reinterpret_cast<const uint4 *>(dst + o);
+            const uint4 cy = *reinterpret_cast<const uint4 *>(dst + o + 64);
+            const __nv_bfloat16 *fr = static_cast<const __nv_bfloat16 *>(a.fresh) +
+                                      static_cast<long long>(t - a.cand0) * a.fresh_stride + h * 128 + pg * 8;
+            s_blk[tb * B + h * 16 + pg] = score_block8(__ldg(reinterpret_cast<const uint4 *>(fr)), cx);
+            s_blk[tb * B + h * 16 + 8 + pg] =
+                score_block8(__ldg(reinterpret_cast<const uint4 *>(fr + 64)), cy);
+        }
+        __syncthreads();
+        for (int tk = threadIdx.x >> 5; tk < TB; tk += kThreads / 32) {
+            const int tt = t0 + tk;
+            if (tt < a.T && tt >= a.cand0 && tt < a.cand0 + a.n_cand) {   // uniform over the warp
+                const float v = reduce_blocks_warp(&s_blk[tk * B], B);
+                if ((threadIdx.x & 31) == 0) a.score_out[tt - a.cand0] = v;
+            }
+        }
+        return;
+    }
     if (a.score_out == nullptr || __ballot_sync(0xFFFFFFFFu, scoring) == 0) return;
     float s1 = 0.0f, s2 = 0.0f;
     if (scoring) {
@@ -413,60 +470,105 @@ __global__ void __launch_bounds__(kThreads, 4) rebase_bf16_kernel(RebaseArgs a, 
     if (scoring && h == 0 && pg == 0) a.score_out[t - a.cand0] = s1;
 }
 
-// fp32: 16 threads per 128-element row, each owning 4 frequency pairs.
+// fp32: 16 threads per 128-element row, each owning 4 frequency pairs.  With the
+// fused score, the CTA whose layer range holds score_layer scores its candidate
+// tokens from the re-based values it holds in registers: each thread's four squared
+// differences of a half form one half of an 8-element block (((q0+q1)+(q2+q3)) from
+// the even thread, ((q4+q5)+(q6+q7)) from the odd one, joined by one shuffle), the
+// block sums meet in shared memory and one warp per token reduces them in the
+// canonical order.
 __global__ void __launch_bounds__(kThreads) rebase_f32_kernel(RebaseArgs a, int layers_per_cta) {
     pdl_wait();   // inputs may come from the previous kernel of the stream
     pdl_trigger();
     __shared__ float4 tab[kMaxTokensPerCta * 64];
     __shared__ int s_delta[kMaxTokensPerCta][3];
+    __shared__ float s_blk[kMaxBlocks];
     const int TB = max(1, (kMaxTokensPerCta / 2) / a.hkv);
     const int t0 = blockIdx.x * TB;
     const int l0 = blockIdx.y * layers_per_cta;
     const int l1 = min(a.n_layers, l0 + layers_per_cta);
     const bool moved_any = build_table(a, t0, TB, s_delta, tab);
-    if (!moved_any && a.in_place) return;
+    const bool cta_scores = a.score_out != nullptr && a.score_layer >= l0 && a.score_layer < l1 &&
+                            t0 < a.cand0 + a.n_cand && t0 + TB > a.cand0;
+    if (!moved_any && a.in_place && !cta_scores) return;   // the same in every thread
 
     const int slot = threadIdx.x;
-    if (slot >= TB * a.hkv * 16) return;
     const int tb = slot / (a.hkv * 16);
     const int h = (slot >> 4) % a.hkv;
     const int pg = slot & 15;
     const int t = t0 + tb;
-    if (t >= a.T) return;
-    const bool moved = (s_delta[tb][0] | s_delta[tb][1] | s_delta[tb][2]) != 0;
-    if (!moved && a.in_place) return;
+    const bool active = slot < TB * a.hkv * 16 && t < a.T;
+    const bool moved = active && (s_delta[tb][0] | s_delta[tb][1] | s_delta[tb][2]) != 0;
+    const bool writes = active && (moved || !a.in_place);
+    const bool scoring = cta_scores && active && t >= a.cand0 && t < a.cand0 + a.n_cand;
     const float *src = static_cast<const float *>(a.k_in);
     float *dst = static_cast<float *>(a.k_out);
     const long long row0 = (static_cast<long long>(t) * a.hkv + h) * 128 + pg * 4;
     const float4 *full = &tab[tb * 64 + pg * 4];
+    float px = 0.0f, py = 0.0f;   // this thread's halves of its two score blocks
     for (int l = l0; l < l1; ++l) {
+        const bool sc = scoring && l == a.score_layer;
+        if (!writes && !sc) continue;
         const long long o = static_cast<long long>(l) * a.layer_stride + row0;
         const float4 x = __ldcs(reinterpret_cast<const float4 *>(src + o));
         const float4 y = __ldcs(reinterpret_cast<const float4 *>(src + o + 64));
-        if (!moved) {
-            __stcs(reinterpret_cast<float4 *>(dst + o), x);
-            __stcs(reinterpret_cast<float4 *>(dst + o + 64), y);
-            continue;
-        }
-        const float xs[4] = {x.x, x.y, x.z, x.w};
-        const float ys[4] = {y.x, y.y, y.z, y.w};
-        float r[4], q[4];
+        float r[4] = {x.x, x.y, x.z, x.w};
+        float q[4] = {y.x, y.y, y.z, y.w};
+        if (moved) {
+            const float xs[4] = {x.x, x.y, x.z, x.w};
+            const float ys[4] = {y.x, y.y, y.z, y.w};
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            const float4 c = full[e];
-            r[e] = rot_f32(xs[e], ys[e], c);
-            q[e] = rot_f32(ys[e], -xs[e], c);
+            for (int e = 0; e < 4; ++e) {
+                const float4 c = full[e];
+                r[e] = rot_f32(xs[e], ys[e], c);
+                q[e] = rot_f32(ys[e], -xs[e], c);
+            }
         }
-        __stcs(reinterpret_cast<float4 *>(dst + o), make_float4(r[0], r[1], r[2], r[3]));
-        __stcs(reinterpret_cast<float4 *>(dst + o + 64), make_float4(q[0], q[1], q[2], q[3]));
+        if (writes) {
+            __stcs(reinterpret_cast<float4 *>(dst + o), make_float4(r[0], r[1], r[2], r[3]));
+            __stcs(reinterpret_cast<float4 *>(dst + o + 64), make_float4(q[0], q[1], q[2], q[3]));
+        }
+        if (sc) {
+            const float *fr = static_cast<const float *>(a.fresh) +
+                              static_cast<long long>(t - a.cand0) * a.fresh_stride + h * 128 + pg * 4;
+            const float4 fx = __ldg(reinterpret_cast<const float4 *>(fr));
+            const float4 fy = __ldg(reinterpret_cast<const float4 *>(fr + 64));
+            const float f1[4] = {fx.x, fx.y, fx.z, fx.w}, f2[4] = {fy.x, fy.y, fy.z, fy.w};
+            float d1[4], d2[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const float u = __fsub_rn(f1[e], r[e]), v = __fsub_rn(f2[e], q[e]);
+                d1[e] = __fmul_rn(u, u);
+                d2[e] = __fmul_rn(v, v);
+            }
+            px = __fadd_rn(__fadd_rn(d1[0], d1[1]), __fadd_rn(d1[2], d1[3]));
+            py = __fadd_rn(__fadd_rn(d2[0], d2[1]), __fadd_rn(d2[2], d2[3]));
+        }
+    }
+    if (!cta_scores) return;   // the same in every thread
+    // block sum = (even thread's half) + (odd thread's half); x + y = y + x exactly
+    const float ox = __shfl_xor_sync(0xFFFFFFFFu, px, 1);
+    const float oy = __shfl_xor_sync(0xFFFFFFFFu, py, 1);
+    const int B = 16 * a.hkv;     // blocks of one token row (TB * B <= kMaxBlocks)
+    if (scoring && (pg & 1) == 0) {
+        s_blk[tb * B + h * 16 + (pg >> 1)] = __fadd_rn(px, ox);
+        s_blk[tb * B + h * 16 + 8 + (pg >> 1)] = __fadd_rn(py, oy);
+    }
+    __syncthreads();
+    for (int tk = threadIdx.x >> 5; tk < TB; tk += kThreads / 32) {
+        const int tt = t0 + tk;
+        if (tt < a.T && tt >= a.cand0 && tt < a.cand0 + a.n_cand) {   // uniform over the warp
+            const float v = reduce_blocks_warp(&s_blk[tk * B], B);
+            if ((threadIdx.x & 31) == 0) a.score_out[tt - a.cand0] = v;
+        }
     }
 }
 
 }  // namespace
 
 bool rebase_fuses_score(const RebaseArgs &a, cs_dtype dt) {
-    // bf16 only, and a token's row must be whole lanes of one warp (8 lanes per head)
-    return dt == CS_DTYPE_BF16 && (a.hkv == 1 || a.hkv == 2 || a.hkv == 4);
+    // every head count the kernels take (bf16 up to 32, fp32 up to 16 kv heads)
+    return (dt == CS_DTYPE_BF16 && a.hkv <= 32) || (dt == CS_DTYPE_F32 && a.hkv <= 16);
 }
 
 cudaError_t launch_rebase(const RebaseArgs &a, cs_dtype dt, cudaStream_t s) {

@@ -130,12 +130,14 @@ __device__ __forceinline__ void find_bin(SelShared *s, int S, uint32_t krem, Get
         s->s_above = 0;
         s->s_cnt = 0;
     }
+    constexpr int kQ = (kBins + kNT - 1) / kNT;   // most bins a thread walks
     const int q = (S + kNT - 1) / kNT;     // bins per thread, walked from the top
     const int hi = S - t * q;              // thread t: bins [hi - q, hi) (clipped at 0)
-    uint32_t v[4] = {0, 0, 0, 0};          // q <= 4 (S <= 2048)
+    uint32_t v[kQ];
     uint32_t mine = 0;
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
+    for (int i = 0; i < kQ; ++i) {
+        v[i] = 0;
         const int j = hi - 1 - i;
         if (i < q && j >= 0) v[i] = get(j);
         mine += v[i];
@@ -145,7 +147,7 @@ __device__ __forceinline__ void find_bin(SelShared *s, int S, uint32_t krem, Get
     if (above < krem && incl >= krem) {
         unsigned long long acc = above;
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
+        for (int i = 0; i < kQ; ++i) {
             if (i < q && acc + v[i] >= krem) {
                 s->s_hit = static_cast<uint32_t>(hi - 1 - i);
                 s->s_above = static_cast<uint32_t>(acc);

@@ -1,7 +1,8 @@
-"""cs_rebase_and_score (steps 1 and 2 in one call) against the two separate calls on the
-same inputs: re-based keys and scores must agree bit for bit, whether the library fuses
-them into one launch (bf16, 1, 2 or 4 kv heads) or runs two; and against the oracle's
-canonical score of the oracle-re-based keys."""
+"""cs_rebase_and_score (steps 1 and 2 in one launch) against the two separate calls on the
+same inputs: re-based keys and scores must agree bit for bit, for every kv head count and
+both storage types (the fused score reduces a token's block sums by lane shuffles when its
+row fits one warp, through shared memory otherwise, and from registers in the fp32
+kernel); and against the oracle's canonical score."""
 import numpy as np
 import pytest
 import torch
@@ -13,10 +14,10 @@ from _helpers import bits16, cuda, f64
 pytestmark = pytest.mark.gpu
 
 
-def _inputs(L, T, H, dtype, seed, n_cand, cand0):
+def _inputs(L, T, H, dtype, seed, n_cand, cand0, sl=1):
     g = torch.Generator().manual_seed(seed)
     k = torch.randn(L, T, H, 128, generator=g).to(dtype)
-    fresh = (k[min(1, L - 1), cand0:cand0 + n_cand].float() +
+    fresh = (k[min(sl, L - 1), cand0:cand0 + n_cand].float() +
              0.3 * torch.randn(n_cand, H, 128, generator=g)).to(dtype)
     loc, glo = W.random_coordinates(T, seed)
     # a third of the tokens do not move (delta 0): their scores are still due
@@ -25,14 +26,18 @@ def _inputs(L, T, H, dtype, seed, n_cand, cand0):
     return k, fresh, loc, glo
 
 
-@pytest.mark.parametrize("H,dtype,in_place", [(1, torch.bfloat16, True), (2, torch.bfloat16, True),
-                                              (4, torch.bfloat16, False), (8, torch.bfloat16, True),
-                                              (2, torch.float32, True)])
-def test_fused_equals_separate_calls(cslib, H, dtype, in_place):
-    L, T, cand0, n_cand = 3, 203, 17, 161
-    k, fresh, loc, glo = _inputs(L, T, H, dtype, 40 + H, n_cand, cand0)
+@pytest.mark.parametrize("H,dtype,in_place,L,sl", [
+    (1, torch.bfloat16, True, 3, 1), (2, torch.bfloat16, True, 3, 1),
+    (4, torch.bfloat16, False, 3, 1), (8, torch.bfloat16, True, 3, 1),
+    (8, torch.bfloat16, False, 6, 5), (3, torch.bfloat16, True, 3, 1),
+    (7, torch.bfloat16, False, 3, 2), (16, torch.bfloat16, True, 2, 1),
+    (1, torch.float32, True, 3, 1), (2, torch.float32, True, 3, 1),
+    (2, torch.float32, False, 6, 5), (3, torch.float32, True, 5, 4),
+    (8, torch.float32, False, 3, 0), (16, torch.float32, True, 2, 1)])
+def test_fused_equals_separate_calls(cslib, H, dtype, in_place, L, sl):
+    T, cand0, n_cand = 203, 17, 161
+    k, fresh, loc, glo = _inputs(L, T, H, dtype, 40 + H, n_cand, cand0, sl)
     pl, pg = cuda(loc), cuda(glo)
-    sl = 1
     # separate calls
     kb = k.cuda()
     cslib.cs_rebase_keys(kb, pl, pg)
@@ -51,7 +56,7 @@ def test_fused_equals_separate_calls(cslib, H, dtype, in_place):
     assert np.array_equal(s_one.cpu().numpy().view(np.uint32), s_sep.cpu().numpy().view(np.uint32))
 
 
-@pytest.mark.parametrize("H", [2, 4])
+@pytest.mark.parametrize("H", [2, 4, 8, 16])
 def test_fused_score_matches_oracle(cslib, H):
     L, T, cand0, n_cand = 2, 140, 40, 100
     k, fresh, loc, glo = _inputs(L, T, H, torch.bfloat16, 70 + H, n_cand, cand0)
@@ -60,6 +65,22 @@ def test_fused_score_matches_oracle(cslib, H):
                                 exp_k[0, cand0:cand0 + n_cand].astype(np.float32))
     _, got = cslib.cs_rebase_and_score(k.cuda(), cuda(loc), cuda(glo), fresh.cuda(), 1, cand0)
     cslib.cs_sync_status()
+    assert np.array_equal(got.cpu().numpy().view(np.uint32), exp.view(np.uint32))
+
+
+@pytest.mark.parametrize("H", [1, 2, 5])
+def test_fused_score_f32_matches_oracle(cslib, H):
+    """fp32 storage: the re-base is within a few ulps of the oracle (not bit for bit), so the
+    score is checked stage-wise: the oracle's canonical score of the keys the GPU re-based,
+    bit for bit, and the keys within the fp32 tolerance of the oracle's rotation."""
+    L, T, cand0, n_cand = 3, 150, 30, 120
+    k, fresh, loc, glo = _inputs(L, T, H, torch.float32, 90 + H, n_cand, cand0)
+    exp_k, _ = O.rebase(f64(k[1])[None], loc, glo, "f32")
+    res, got = cslib.cs_rebase_and_score(k.cuda(), cuda(loc), cuda(glo), fresh.cuda(), 1, cand0)
+    cslib.cs_sync_status()
+    assert np.max(np.abs(f64(res[1]) - exp_k[0])) <= 1e-5
+    exp = O.score_f32_canonical(f64(fresh).astype(np.float32),
+                                f64(res[1, cand0:cand0 + n_cand]).astype(np.float32))
     assert np.array_equal(got.cpu().numpy().view(np.uint32), exp.view(np.uint32))
 
 
