@@ -163,6 +163,38 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(sm)}
 
 
+def numa_nodes() -> int:
+    """NUMA nodes the host exposes (1 if unknown)."""
+    try:
+        return max(1, len([d for d in os.listdir("/sys/devices/system/node")
+                           if d.startswith("node") and d[4:].isdigit()]))
+    except OSError:
+        return 1
+
+
+def host_link_rates(h_in, d_in, h_out, d_out, stream) -> dict:
+    """Host<->device copy rates of the e2e buffers on their own (pinned host memory):
+    one host-to-device copy of the stored keys and one device-to-host copy of the output,
+    each timed with CUDA events, best of 3."""
+    def rate(dst, src):
+        best = None
+        for _ in range(3):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            dst.copy_(src, non_blocking=True)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            ms = e0.elapsed_time(e1)
+            best = ms if best is None else min(best, ms)
+        return round(src.numel() * src.element_size() / (best / 1e3) / 1e9, 1)
+    return {"h2d_gbs": rate(d_in, h_in), "d2h_gbs": rate(h_out, d_out),
+            "h2d_bytes": h_in.numel() * h_in.element_size(),
+            "d2h_bytes": d_out.numel() * d_out.element_size(),
+            "pinned": bool(h_in.is_pinned()), "host_numa_nodes": numa_nodes(),
+            "placement": "pinned with cudaHostAlloc through torch on the process's NUMA node "
+                         "(the host exposes the node count given)"}
+
+
 def config_of(w, ws: int) -> dict:
     """The workload description both arms print (the same dict for the same run)."""
     return {"workload": w.name, "layers": w.n_layers, "chunks": w.n_chunks,
@@ -375,6 +407,7 @@ def run_gpu(args, w, ws, rank, local):
     pipe_mean = time_e2e(pipelined.replay)
     pipe_spread = spread[pipelined.replay]
     cs.cs_sync_status()
+    link = host_link_rates(host["k"], x["k"], out_host["o"], q.out, stream)
     e2e_mean = max_over_ranks(pipe_mean, dev)
     graph_mean = max_over_ranks(graph_mean, dev)
     eager_mean = max_over_ranks(eager_mean, dev)
@@ -387,7 +420,8 @@ def run_gpu(args, w, ws, rank, local):
                    "path": "PipelinedQuery.replay (copies and kernels overlapped by layer "
                            "group, one CUDA graph)",
                    "graph_value": round(replica_throughput(w.t_vis, graph_mean, ws), 1),
-                   "eager_value": round(replica_throughput(w.t_vis, eager_mean, ws), 1)}
+                   "eager_value": round(replica_throughput(w.t_vis, eager_mean, ws), 1),
+                   "host_link": link}
     # the CPU-baseline leg reads the GPU arm's own inputs (not its results)
     return line, x, pristine
 

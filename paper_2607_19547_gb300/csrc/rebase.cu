@@ -17,6 +17,7 @@
 // double-float and rounds that.  fp32 outputs always use the double-float
 // result.
 #include <algorithm>
+#include <mutex>
 
 #include "cs_device.cuh"
 #include "cs_internal.h"
@@ -98,7 +99,7 @@ __device__ __forceinline__ uint32_t rot_bf16_df(float u, float w, float4 cs4) {
 // memory (their raw input words and where they came from) and are redone by the
 // whole warp together, one output pair per lane, so the rare slow path never runs
 // on one lane while the other 31 wait.
-constexpr int kQueue = 64;   // entries per warp
+constexpr int kQueue = 48;   // entries per warp
 
 __shared__ uint4 q_xy[kThreads / 32][2 * kQueue];   // first- and second-half words
 __shared__ uint32_t q_meta[kThreads / 32][kQueue];  // (slice index << 5) | owning lane
@@ -142,6 +143,32 @@ __device__ __forceinline__ uint32_t pack_bf16x2_rn(float lo, float hi) {
     uint32_t r;
     asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
     return r;
+}
+
+// Per-thread staging of the next layers' input words in shared memory with 16-byte
+// asynchronous copies (cp.async, bypassing L1): kStages layers of every thread's two
+// words are in flight without holding registers.  Each thread copies and later reads
+// only its own slots, so the copies need no block barrier: a wait on the thread's own
+// copy groups makes them visible to it.  Slot (stage s, half h) of thread x sits at
+// word (s * 2 + h) * kThreads + x, so a warp's reads and copies touch consecutive
+// 16-byte words.
+constexpr int kStages = 4;
+constexpr size_t kStageBytes = static_cast<size_t>(kStages) * 2 * kThreads * 16;
+
+__device__ __forceinline__ uint4 *stage_slot(uint4 *buf, int s, int h) {
+    return buf + (s * 2 + h) * kThreads + threadIdx.x;
+}
+__device__ __forceinline__ void cp_async16(uint4 *smem, const void *gmem) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(smem)), "l"(gmem)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+    asm volatile("cp.async.commit_group;" ::: "memory");
+}
+// Waits until at most kStages - 1 of this thread's copy groups are still in flight
+// (groups complete in order, so every older group is complete).
+__device__ __forceinline__ void cp_async_wait_stage() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(kStages - 1) : "memory");
 }
 
 // fp32 result of u*c - w*s from the double-float evaluation (an overflowing
@@ -292,20 +319,27 @@ __device__ __forceinline__ float reduce_blocks_warp(const float *blk, int B) {
 
 // The streaming part of the bf16 kernel for one thread's slices (see the kernel
 // below).  `part` holds the lanes of this warp that rotate (moved tokens with
-// layers to walk); they all walk the same number of layers.
+// layers to walk); they all walk the same number of layers.  The first kStages
+// layers' words were requested by the kernel (stage_first); every iteration waits
+// for its stage, uses it, and requests the layer kStages further on into it.
 __device__ __forceinline__ void stream_slices(const __nv_bfloat16 *src, __nv_bfloat16 *dst,
                                               long long obase, long long lstep, int count,
                                               bool moved, unsigned part, int trow,
-                                              const float4 *tab, uint4 xv, uint4 yv) {
+                                              const float4 *tab, uint4 *stage) {
+    int s = 0;   // stage holding layer i
     if (!moved) {   // out-of-place copy of an unmoved token
         for (int i = 0; i < count; ++i) {
+            cp_async_wait_stage();
+            const uint4 xv = *stage_slot(stage, s, 0), yv = *stage_slot(stage, s, 1);
             const long long o = obase + i * lstep;
-            if (i > 0) {
-                xv = __ldcs(reinterpret_cast<const uint4 *>(src + o));
-                yv = __ldcs(reinterpret_cast<const uint4 *>(src + o + 64));
-            }
             __stcs(reinterpret_cast<uint4 *>(dst + o), xv);
             __stcs(reinterpret_cast<uint4 *>(dst + o + 64), yv);
+            if (i + kStages < count) {
+                cp_async16(stage_slot(stage, s, 0), src + o + kStages * lstep);
+                cp_async16(stage_slot(stage, s, 1), src + o + kStages * lstep + 64);
+            }
+            cp_async_commit();
+            s = s + 1 == kStages ? 0 : s + 1;
         }
         return;
     }
@@ -323,15 +357,12 @@ __device__ __forceinline__ void stream_slices(const __nv_bfloat16 *src, __nv_bfl
             redo_queue(queued, part, obase, lstep, trow, tab, dst);
             queued = 0;
         }
-        uint4 xn = make_uint4(0, 0, 0, 0), yn = make_uint4(0, 0, 0, 0);
-        if (i + 1 < count) {
-            xn = __ldcs(reinterpret_cast<const uint4 *>(src + obase + (i + 1) * lstep));
-            yn = __ldcs(reinterpret_cast<const uint4 *>(src + obase + (i + 1) * lstep + 64));
-        }
+        cp_async_wait_stage();
+        const uint4 xv = *stage_slot(stage, s, 0), yv = *stage_slot(stage, s, 1);
         uint32_t ow[4], pw[4];
         const bool ok = rotate_slice(xv, yv, c, sn, ow, pw);
+        const long long o = obase + i * lstep;
         if (ok) {
-            const long long o = obase + i * lstep;
             __stcs(reinterpret_cast<uint4 *>(dst + o), make_uint4(ow[0], ow[1], ow[2], ow[3]));
             __stcs(reinterpret_cast<uint4 *>(dst + o + 64), make_uint4(pw[0], pw[1], pw[2], pw[3]));
         }
@@ -346,8 +377,14 @@ __device__ __forceinline__ void stream_slices(const __nv_bfloat16 *src, __nv_bfl
             }
             queued += __popc(fails);
         }
-        xv = xn;
-        yv = yn;
+        // the stage's words have been used (stored or queued): request the layer kStages
+        // further on into it
+        if (i + kStages < count) {
+            cp_async16(stage_slot(stage, s, 0), src + o + kStages * lstep);
+            cp_async16(stage_slot(stage, s, 1), src + o + kStages * lstep + 64);
+        }
+        cp_async_commit();
+        s = s + 1 == kStages ? 0 : s + 1;
     }
     if (queued) redo_queue(queued, part, obase, lstep, trow, tab, dst);
 }
@@ -407,10 +444,14 @@ __global__ void __launch_bounds__(kThreads, 4) rebase_bf16_kernel(RebaseArgs a, 
     const long long row0 = (static_cast<long long>(t) * hkv + h) * 128 + pg * 8;
     const long long lstep = static_cast<long long>(n_slots) * a.layer_stride;
     const long long obase = static_cast<long long>(lfirst) * a.layer_stride + row0;
-    uint4 xv = make_uint4(0, 0, 0, 0), yv = make_uint4(0, 0, 0, 0);
-    if (count > 0) {
-        xv = __ldcs(reinterpret_cast<const uint4 *>(src + obase));
-        yv = __ldcs(reinterpret_cast<const uint4 *>(src + obase + 64));
+    // the first layers' words go out before the table is built (empty groups past count)
+    extern __shared__ uint4 stage[];
+    for (int st = 0; st < kStages; ++st) {
+        if (st < count) {
+            cp_async16(stage_slot(stage, st, 0), src + obase + st * lstep);
+            cp_async16(stage_slot(stage, st, 1), src + obase + st * lstep + 64);
+        }
+        cp_async_commit();
     }
     const bool moved_any = build_table(a, t0, TB, s_delta, tab);
     const bool scoring = a.score_out != nullptr && slot < n_slots && t < a.T && t >= a.cand0 &&
@@ -419,7 +460,7 @@ __global__ void __launch_bounds__(kThreads, 4) rebase_bf16_kernel(RebaseArgs a, 
     // build_table ended with a block barrier: every lane takes part in this ballot
     const unsigned part = __ballot_sync(0xFFFFFFFFu, count > 0 && moved && moved_any);
     if (count > 0)
-        stream_slices(src, dst, obase, lstep, count, moved, part, tb * 64 + pg * 8, tab, xv, yv);
+        stream_slices(src, dst, obase, lstep, count, moved, part, tb * 64 + pg * 8, tab, stage);
     if (HKV == 0) {
         // any head count: a token's row may span several warps, so its block sums meet in
         // shared memory and one warp per token reduces them in the canonical order
@@ -589,7 +630,18 @@ cudaError_t launch_rebase(const RebaseArgs &a, cs_dtype dt, cudaStream_t s) {
         dim3 grid(blocks, (a.n_layers + l_per_cta - 1) / l_per_cta);
         auto *kern = a.hkv == 1 ? rebase_bf16_kernel<1> : a.hkv == 2 ? rebase_bf16_kernel<2>
                    : a.hkv == 4 ? rebase_bf16_kernel<4> : rebase_bf16_kernel<0>;
-        return launch_pdl(kern, grid, dim3(kThreads), 0, s, a, TB, l_per_cta);
+        static std::once_flag attr_once;
+        static cudaError_t attr_err = cudaSuccess;
+        std::call_once(attr_once, [] {
+            for (auto *k : {rebase_bf16_kernel<1>, rebase_bf16_kernel<2>, rebase_bf16_kernel<4>,
+                            rebase_bf16_kernel<0>}) {
+                const cudaError_t e = cudaFuncSetAttribute(
+                    k, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kStageBytes));
+                if (e != cudaSuccess) attr_err = e;
+            }
+        });
+        if (attr_err != cudaSuccess) return attr_err;
+        return launch_pdl(kern, grid, dim3(kThreads), kStageBytes, s, a, TB, l_per_cta);
     } else {
         const int TB = a.hkv >= kMaxTokensPerCta / 2 ? 1 : (kMaxTokensPerCta / 2) / a.hkv;
         const int layers_per_cta = 4;
