@@ -11,11 +11,12 @@
 //   - up to three MSB-first passes over 11-, 11- and 10-bit digits find K*, the
 //     k-th largest key, and how many keys equal to K* are taken (the lowest-index
 //     ones).  A pass: every CTA counts its own keys that match the digits resolved
-//     so far into a 2048-bin histogram in its shared memory; after a cluster
-//     barrier CTA r sums bin slice r (2048/C bins) over all C histograms through
-//     distributed shared memory; after a second barrier every CTA reads the C
-//     slice totals and the one slice that holds the k-th key and takes the same
-//     decision.  The histogram is double-buffered by pass parity, so a CTA never
+//     so far into a 2048-bin histogram in its shared memory and sums it over 64
+//     groups of 32 bins; after one cluster barrier every CTA reads the C x 64 group
+//     sums through distributed shared memory (spread over its threads), finds the
+//     group that holds the k-th key with a warp-wide scan, then reads that group's
+//     32 bins from the C CTAs and finds the bin the same way.  Every CTA takes the
+//     same decision from the same counts.  The histograms are double-buffered by pass parity, so a CTA never
 //     clears a buffer that another CTA may still read.  The passes stop once every
 //     key left in K*'s bin is taken;
 //   - one block-wide scan of the per-thread (greater, equal) counts, plus the
@@ -37,6 +38,8 @@ namespace {
 constexpr int kNT = 512;          // threads per CTA
 constexpr int kWarps = kNT / 32;
 constexpr int kBins = 2048;
+constexpr int kFine = 32;                  // bins per group
+constexpr int kGroups = kBins / kFine;     // 64 groups
 constexpr int kMaxCluster = 16;
 
 // Order-preserving key of an fp32 bit pattern u (scores are read as raw 32-bit
@@ -106,58 +109,24 @@ __device__ __forceinline__ T block_incl_scan(T v, T *wsum) {
 }
 
 struct SelShared {
-    uint32_t hist[2][kBins];            // per-pass histograms (double-buffered)
-    uint32_t red[kBins];                // this CTA's reduced bin slice (C > 1)
-    uint32_t part[kNT];                 // partial sums of the slice reduction
-    uint32_t wtot[kWarps];              // per-warp sums of the slice total
+    uint32_t hist[2][kBins];            // per-pass histograms (double-buffered by pass parity)
+    uint32_t coarse[2][kGroups];        // their sums over groups of kFine consecutive bins
     unsigned long long wsum[kWarps];    // block scan scratch
     unsigned long long cta_counts;      // this CTA's (greater << 32 | equal) in the final phase
-    uint32_t slice_total;               // sum of red[]
-    uint32_t s_digit, s_krem, s_done;   // the pass's decision
-    uint32_t s_hit, s_above, s_cnt;     // bin search result inside the block
     unsigned long long s_before;        // counts of the CTAs before this one
+    uint32_t part[kNT];                 // per-thread partial sums of a decision step
+    uint32_t s_group, s_above, s_hit, s_cnt;   // the pass's decision
 };
 
-// Finds, among S bin counts read through get(j) (j = 0..S-1, ascending digits), the
-// bin that holds the krem-th largest key: sets s->s_hit = that bin, s->s_above = the
-// keys in higher bins and s->s_cnt = the keys in that bin.  Every thread calls it (it
-// contains block barriers).
-template <typename Get>
-__device__ __forceinline__ void find_bin(SelShared *s, int S, uint32_t krem, Get get) {
-    const int t = threadIdx.x;
-    if (t == 0) {   // defined results even if no bin were found (the counts rule it out)
-        s->s_hit = 0;
-        s->s_above = 0;
-        s->s_cnt = 0;
-    }
-    constexpr int kQ = (kBins + kNT - 1) / kNT;   // most bins a thread walks
-    const int q = (S + kNT - 1) / kNT;     // bins per thread, walked from the top
-    const int hi = S - t * q;              // thread t: bins [hi - q, hi) (clipped at 0)
-    uint32_t v[kQ];
-    uint32_t mine = 0;
+// Inclusive scan over the 32 lanes of a warp.
+__device__ __forceinline__ uint32_t warp_incl_scan(uint32_t v) {
+    const int lane = threadIdx.x & 31;
 #pragma unroll
-    for (int i = 0; i < kQ; ++i) {
-        v[i] = 0;
-        const int j = hi - 1 - i;
-        if (i < q && j >= 0) v[i] = get(j);
-        mine += v[i];
+    for (int o = 1; o < 32; o *= 2) {
+        const uint32_t y = __shfl_up_sync(0xFFFFFFFFu, v, o);
+        if (lane >= o) v += y;
     }
-    const unsigned long long incl = block_incl_scan<unsigned long long>(mine, s->wsum);
-    const unsigned long long above = incl - mine;
-    if (above < krem && incl >= krem) {
-        unsigned long long acc = above;
-#pragma unroll
-        for (int i = 0; i < kQ; ++i) {
-            if (i < q && acc + v[i] >= krem) {
-                s->s_hit = static_cast<uint32_t>(hi - 1 - i);
-                s->s_above = static_cast<uint32_t>(acc);
-                s->s_cnt = v[i];
-                break;
-            }
-            acc += v[i];
-        }
-    }
-    __syncthreads();
+    return v;
 }
 
 // KPT > 0: exactly KPT keys per thread in registers (per == KPT); KPT == 0: `per`
@@ -223,108 +192,96 @@ select_kernel(const uint32_t *__restrict__ score, int n, int k, int idx_base, in
     };
 
     for (int j = t; j < 2 * kBins; j += kNT) (&s->hist[0][0])[j] = 0u;
+    if (t < 2 * kGroups) (&s->coarse[0][0])[t] = 0u;
     __syncthreads();
 
-    const int S = kBins / static_cast<int>(C);   // bins of one slice
+    // a word of this CTA's shared memory as seen in CTA c of the cluster (c == r: itself)
+    auto rd = [&](const uint32_t *p, uint32_t c) -> uint32_t {
+        return C == 1 ? *p : dsmem_ld(dsmem_addr(p, c));
+    };
+    const int lane = t & 31, warp = t >> 5;
     uint32_t prefix = 0, pmask = 0, krem = static_cast<uint32_t>(k);
 #pragma unroll 1
     for (int pass = 0; pass < 3; ++pass) {
         const int shift = pass == 0 ? 21 : (pass == 1 ? 10 : 0);
         const uint32_t dmask = pass == 2 ? 0x3FFu : 0x7FFu;
         uint32_t *hist = s->hist[pass & 1];
+        uint32_t *coarse = s->coarse[pass & 1];
         for_keys([&](int, uint32_t key) {
             if ((key & pmask) == prefix) atomicAdd(&hist[(key >> shift) & dmask], 1u);
         });
-        uint32_t digit, above;
-        if (C == 1) {
-            __syncthreads();
-            find_bin(s, kBins, krem, [&](int j) { return hist[j]; });
-            digit = s->s_hit;
-            above = s->s_above;
-            // the other buffer is cleared for the next pass (nobody else reads it)
-            for (int j = t; j < kBins; j += kNT) s->hist[(pass + 1) & 1][j] = 0u;
-        } else {
-            cluster_sync();
-            // every CTA has finished reading the other buffer (last pass): clear it
-            for (int j = t; j < kBins; j += kNT) s->hist[(pass + 1) & 1][j] = 0u;
-            // reduce bin slice r over the C histograms of the cluster
-            uint32_t tot = 0;
-            if (S >= kNT) {
-                for (int bl = t; bl < S; bl += kNT) {
-                    uint32_t v = 0;
-                    for (uint32_t src = 0; src < C; ++src)
-                        v += dsmem_ld(dsmem_addr(&hist[r * S + bl], src));
-                    s->red[bl] = v;
-                    tot += v;
-                }
-            } else {
-                const int G = kNT / S, per_src = static_cast<int>(C) / G;
-                const int bl = t % S, g = t / S;
-                uint32_t v = 0;
-                for (int m = 0; m < per_src; ++m)
-                    v += dsmem_ld(dsmem_addr(&hist[r * S + bl], static_cast<uint32_t>(g * per_src + m)));
-                s->part[t] = v;
-                __syncthreads();
-                if (t < S) {
-                    uint32_t w = 0;
-                    for (int gg = 0; gg < G; ++gg) w += s->part[t + gg * S];
-                    s->red[t] = w;
-                    tot = w;
-                }
-            }
-            // slice total
-#pragma unroll
-            for (int o = 16; o >= 1; o /= 2) tot += __shfl_xor_sync(0xFFFFFFFFu, tot, o);
-            if ((t & 31) == 0) s->wtot[t >> 5] = tot;
-            __syncthreads();
-            if (t == 0) {
-                uint32_t a = 0;
-                for (int w = 0; w < kWarps; ++w) a += s->wtot[w];
-                s->slice_total = a;
-            }
-            cluster_sync();
-            // the slice holding the k-th key: slices of higher rank hold higher digits
-            if (t == 0) {
-                s->s_digit = 0;
-                s->s_above = 0;
-            }
-            __syncthreads();
-            if (t < 32) {
-                const uint32_t tj = static_cast<uint32_t>(t) < C
-                                        ? dsmem_ld(dsmem_addr(&s->slice_total, static_cast<uint32_t>(t)))
-                                        : 0u;
-                // inclusive sum over slices >= t (from the top)
-                uint32_t incl = tj;
-#pragma unroll
-                for (int o = 1; o < 32; o *= 2) {
-                    const uint32_t y = __shfl_down_sync(0xFFFFFFFFu, incl, o);
-                    if (t + o < 32) incl += y;
-                }
-                const uint32_t abv = incl - tj;
-                if (static_cast<uint32_t>(t) < C && abv < krem && incl >= krem) {
-                    s->s_digit = static_cast<uint32_t>(t);   // the slice
-                    s->s_above = abv;
-                }
-            }
-            __syncthreads();
-            // (the counts guarantee a slice is found; the clamp keeps every remote
-            // address inside the cluster regardless)
-            const uint32_t sl = min(s->s_digit, C - 1u), above_sl = s->s_above;
-            __syncthreads();   // s_above is rewritten by find_bin
-            find_bin(s, S, krem - above_sl,
-                     [&](int j) { return dsmem_ld(dsmem_addr(&s->red[j], sl)); });
-            digit = sl * static_cast<uint32_t>(S) + s->s_hit;
-            above = above_sl + s->s_above;
+        __syncthreads();
+        {   // group sums: thread t sums bins 4t..4t+3, eight threads make a group of 32
+            const uint4 h4 = reinterpret_cast<const uint4 *>(hist)[t];
+            uint32_t v = h4.x + h4.y + h4.z + h4.w;
+            v += __shfl_xor_sync(0xFFFFFFFFu, v, 4);
+            v += __shfl_xor_sync(0xFFFFFFFFu, v, 2);
+            v += __shfl_xor_sync(0xFFFFFFFFu, v, 1);
+            if ((t & 7) == 0) coarse[t >> 3] = v;
         }
-        // digit holds the k-th largest key among those with the resolved prefix; when
+        if (C > 1) {
+            cluster_sync();
+        } else {
+            __syncthreads();
+        }
+        // every CTA has finished reading the other buffers (last pass): clear them
+        for (int j = t; j < kBins; j += kNT) s->hist[(pass + 1) & 1][j] = 0u;
+        if (t < kGroups) s->coarse[(pass + 1) & 1][t] = 0u;
+        {   // cluster-wide group sums: thread t adds group t % 64 of CTAs t / 64, t / 64 + 8, ...
+            uint32_t v = 0;
+            for (uint32_t c = static_cast<uint32_t>(t / kGroups); c < C; c += kNT / kGroups)
+                v += rd(&coarse[t % kGroups], c);
+            s->part[t] = v;
+        }
+        __syncthreads();
+        if (warp == 0) {
+            // lane l holds groups 63 - 2l and 62 - 2l: lane order is descending digit order
+            uint32_t ga = 0, gb = 0;
+#pragma unroll
+            for (int m = 0; m < kNT / kGroups; ++m) {
+                ga += s->part[(kGroups - 1 - 2 * lane) + kGroups * m];
+                gb += s->part[(kGroups - 2 - 2 * lane) + kGroups * m];
+            }
+            const uint32_t incl = warp_incl_scan(ga + gb);
+            const uint32_t above = incl - ga - gb;
+            if (above < krem && incl >= krem) {
+                const bool hi = above + ga >= krem;
+                s->s_group = static_cast<uint32_t>(hi ? kGroups - 1 - 2 * lane : kGroups - 2 - 2 * lane);
+                s->s_above = hi ? above : above + ga;
+            }
+        }
+        __syncthreads();
+        const uint32_t grp = min(s->s_group, static_cast<uint32_t>(kGroups - 1));
+        const uint32_t above_g = s->s_above;
+        {   // the group's 32 bins in every CTA: thread t reads bin t % 32 of CTA t / 32
+            const uint32_t c = static_cast<uint32_t>(t / kFine);
+            s->part[t] = c < C ? rd(&hist[grp * kFine + lane], c) : 0u;
+        }
+        __syncthreads();
+        if (warp == 0) {
+            // lane l holds bin 31 - l of the group (descending digit order)
+            uint32_t f = 0;
+#pragma unroll
+            for (int c = 0; c < kNT / kFine; ++c) f += s->part[(kFine - 1 - lane) + kFine * c];
+            const uint32_t incl = warp_incl_scan(f);
+            const uint32_t above = incl - f, want = krem - above_g;
+            if (above < want && incl >= want) {
+                s->s_hit = grp * kFine + static_cast<uint32_t>(kFine - 1 - lane);
+                s->s_above = above_g + above;
+                s->s_cnt = f;
+            }
+        }
+        __syncthreads();
+        // the digit of the k-th largest key among those with the resolved prefix; when
         // every key left in its bin is taken the remaining digits cannot change the
         // selection
-        const uint32_t krem_new = krem - above;
+        const uint32_t digit = s->s_hit;
+        const uint32_t krem_new = krem - s->s_above;
         const bool done = s->s_cnt == krem_new;
         prefix |= digit << shift;
         pmask |= dmask << shift;
         krem = krem_new;
-        __syncthreads();   // s_hit / s_above / s_digit are rewritten in the next pass
+        __syncthreads();   // the decision words are rewritten in the next pass
         if (done) break;   // uniform across the cluster: every CTA took the same decision
     }
 
@@ -353,7 +310,9 @@ select_kernel(const uint32_t *__restrict__ score, int n, int k, int idx_base, in
         }
         __syncthreads();
         before_cta = s->s_before;
-        cluster_arrive();   // this CTA reads no other CTA's shared memory after this point
+        // this CTA reads no other CTA's shared memory after this point; the wait at the
+        // end keeps its own alive until every CTA has read it
+        asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
     }
     const unsigned long long before = before_cta + before_t;
     const uint32_t gt_before = static_cast<uint32_t>(before >> 32);
