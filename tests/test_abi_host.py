@@ -138,6 +138,14 @@ def test_attention_rejects_bad_arguments(cslib):
     assert "overlaps" in cslib.cs_last_error_detail()
     assert call(Hq=256, Hkv=1) == cslib.CS_ERR_UNSUPPORTED
     assert call(M=0, q=None, o=None) == cslib.CS_OK
+    # the optional LSE: 4-byte aligned, and not over k, v (read by other CTAs) or o
+    far = FAKE + (1 << 24)
+    assert call(o=far, lse=far + (1 << 20) + 2) == cslib.CS_ERR_INVALID_ARG
+    assert "aligned" in cslib.cs_last_error_detail()
+    assert call(o=far, lse=FAKE + 64) == cslib.CS_ERR_INVALID_ARG
+    assert "lse overlaps k or v" in cslib.cs_last_error_detail()
+    assert call(o=far, lse=far + 256) == cslib.CS_ERR_INVALID_ARG
+    assert "lse overlaps o" in cslib.cs_last_error_detail()
 
 
 def test_debug_wait_rejects_bad_limits(cslib):

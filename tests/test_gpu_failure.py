@@ -30,3 +30,17 @@ def test_bounded_wait_times_out_and_context_survives(cslib):
     cslib.cs_sync_status()
     exp, _ = O.rebase(before, loc, glo, "bf16")
     assert np.array_equal(f64(k), exp)
+
+
+def test_status_record_is_device_wide_and_taken_once(cslib):
+    """An error recorded by a kernel on one stream is reported by the next take on any
+    stream of the device (the record is device-wide), exactly once."""
+    cslib.cs_sync_status()
+    a, b = torch.cuda.Stream(), torch.cuda.Stream()
+    cslib.cs_debug_wait_timeout(20000, stream=a)   # records CS_ERR_TIMEOUT on stream a
+    a.synchronize()
+    with pytest.raises(cslib.CsError) as e:
+        cslib.cs_sync_status(stream=b)
+    assert e.value.status == cslib.CS_ERR_TIMEOUT
+    cslib.cs_sync_status(stream=a)                  # taken already: nothing left
+    cslib.cs_sync_status(stream=b)
