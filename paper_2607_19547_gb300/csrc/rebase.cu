@@ -257,10 +257,13 @@ __device__ __forceinline__ bool rotate_slice(const uint4 &xv, const uint4 &yv, c
         const int e0 = 2 * w, e1 = 2 * w + 1;
         const float x0 = bf16_lo(xw[w]), x1 = bf16_hi(xw[w]);
         const float y0 = bf16_lo(yw[w]), y1 = bf16_hi(yw[w]);
-        const float2 r1 = make_float2(__fmaf_rn(x0, c[e0], -__fmul_rn(y0, sn[e0])),    // x c - y s
-                                      __fmaf_rn(x1, c[e1], -__fmul_rn(y1, sn[e1])));
-        const float2 r2 = make_float2(__fmaf_rn(y0, c[e0], __fmul_rn(x0, sn[e0])),     // y c + x s
-                                      __fmaf_rn(y1, c[e1], __fmul_rn(x1, sn[e1])));
+        // two frequency pairs at once in packed fp32 (the same roundings as one pair at a
+        // time: one product, then one fused multiply-add)
+        const float2 X = make_float2(x0, x1), Y = make_float2(y0, y1);
+        const float2 C = make_float2(c[e0], c[e1]), S = make_float2(sn[e0], sn[e1]);
+        const float2 ys = __fmul2_rn(Y, S), xs = __fmul2_rn(X, S);
+        const float2 r1 = __ffma2_rn(X, C, make_float2(-ys.x, -ys.y));   // x c - y s
+        const float2 r2 = __ffma2_rn(Y, C, xs);                          // y c + x s
         const float2 u = make_float2(__fadd_rn(fabsf(x0), fabsf(y0)), __fadd_rn(fabsf(x1), fabsf(y1)));
         const float2 E = __ffma2_rn(u, kE, kT);
         const float2 lo1 = __ffma2_rn(E, kM, r1), hi1 = __fadd2_rn(r1, E);
