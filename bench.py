@@ -619,9 +619,11 @@ class OracleSample:
         w = self.w
         return (f"re-base of layer(s) {self.layers} of {w.n_layers} (all {w.T} tokens, scaled by "
                 f"{w.n_layers}/{len(self.layers)}); score and select over all {w.n_cand} "
-                f"candidates; attention of {min(n_rows, w.M)} of {w.M} query rows (seeded, first "
-                f"and last included) at those layers, scaled by {w.n_layers}/{len(self.layers)} "
-                f"x sum(qpos+1) over all rows / over the sampled rows; numpy fp64")
+                f"candidates (timed in full); attention of {min(n_rows, w.M)} of {w.M} query rows "
+                f"(seeded, first and last included) at those layers, scaled by "
+                f"{w.n_layers}/{len(self.layers)} x sum(qpos+1) over all rows / over the sampled "
+                f"rows; the full-step time and the rate are extrapolated from this sample; "
+                f"numpy fp64")
 
     def rate(self, workers: int, steps: int, n_rows: int, seed0: int = 0):
         """(tokens/s of the estimated full step, per-step timing dicts)."""
@@ -648,6 +650,7 @@ def cpu_baseline(w, x, layers, n_rows):
             "cpu_model": cpu_model(),
             "sampled_s": round(tn[0]["sampled_s"], 3),
             "full_step_s_est": round(tn[0]["full_step_s_est"], 3),
+            "value_is": "extrapolated from the sampled step",
             "single_thread": {"value": round(r1, 2), "unit": UNIT, "cores": 1,
                               "sampled_s": round(t1[0]["sampled_s"], 3),
                               "full_step_s_est": round(t1[0]["full_step_s_est"], 3)}}
@@ -680,6 +683,7 @@ def run_reference(args, w, ws):
             "ms_per_step_is": "wall time of one sampled step as run (the timed region is "
                               "steps x this); value is T_vis / the estimated full-step time",
             "full_step_ms_est": round(1e3 * full, 3),
+            "value_is": "extrapolated from the sampled steps (see cpu_baseline.sample)",
             "wall_s_timed_loop": round(wall, 3),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": DATA + " (CPU generator)", "config": config_of(w, ws),
