@@ -558,12 +558,9 @@ cs_status launch_attn_tc(const AttnArgs &a, cudaStream_t s) {
     p.qpos = a.qpos;
     p.status = a.status;
     const size_t smem = Smem::total + 1024;
-    static std::once_flag attr_once;
-    static cudaError_t attr_err = cudaSuccess;
-    std::call_once(attr_once, [&] {
-        attr_err = cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                        static_cast<int>(smem));
-    });
+    const cudaError_t attr_err = func_attr_once(reinterpret_cast<const void *>(attn_tc_kernel),
+                                                cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                static_cast<int>(smem));
     if (attr_err != cudaSuccess) return cuda_fail(attr_err, "cudaFuncSetAttribute");
     attn_tc_kernel<<<static_cast<unsigned>(items), kThreads, smem, s>>>(tq, tk, tv, to, p);
     const cudaError_t e = cudaGetLastError();

@@ -113,6 +113,28 @@ unsigned int *status_word() {
     return g_status_addr[dev];
 }
 
+cudaError_t func_attr_once(const void *fn, cudaFuncAttribute attr, int value) {
+    struct Entry {
+        const void *fn;
+        int dev;
+        int attr;
+        cudaError_t err;
+    };
+    static std::mutex mu;
+    static Entry done[64];
+    static int n_done = 0;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    std::lock_guard<std::mutex> lock(mu);
+    for (int i = 0; i < n_done; ++i)
+        if (done[i].fn == fn && done[i].dev == dev && done[i].attr == static_cast<int>(attr))
+            return done[i].err;
+    e = cudaFuncSetAttribute(fn, attr, value);
+    if (n_done < 64) done[n_done++] = Entry{fn, dev, static_cast<int>(attr), e};
+    return e;
+}
+
 int sm_count() {
     int dev = 0, n = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return 0;

@@ -22,6 +22,11 @@ unsigned int *status_word();
 // Number of SMs of the current device (0 if it cannot be queried).
 int sm_count();
 
+// Sets a function attribute of `fn` on the current device, once per (function, device):
+// function attributes belong to the device's context, so a process that drives several
+// devices sets them on each.  Returns the (first) result.
+cudaError_t func_attr_once(const void *fn, cudaFuncAttribute attr, int value);
+
 // Records a detail string for cs_last_error_detail and returns `s`.
 cs_status fail(cs_status s, const char *fmt, ...);
 cs_status cuda_fail(cudaError_t e, const char *what);

@@ -17,7 +17,6 @@
 // double-float and rounds that.  fp32 outputs always use the double-float
 // result.
 #include <algorithm>
-#include <mutex>
 
 #include "cs_device.cuh"
 #include "cs_internal.h"
@@ -633,16 +632,9 @@ cudaError_t launch_rebase(const RebaseArgs &a, cs_dtype dt, cudaStream_t s) {
         dim3 grid(blocks, (a.n_layers + l_per_cta - 1) / l_per_cta);
         auto *kern = a.hkv == 1 ? rebase_bf16_kernel<1> : a.hkv == 2 ? rebase_bf16_kernel<2>
                    : a.hkv == 4 ? rebase_bf16_kernel<4> : rebase_bf16_kernel<0>;
-        static std::once_flag attr_once;
-        static cudaError_t attr_err = cudaSuccess;
-        std::call_once(attr_once, [] {
-            for (auto *k : {rebase_bf16_kernel<1>, rebase_bf16_kernel<2>, rebase_bf16_kernel<4>,
-                            rebase_bf16_kernel<0>}) {
-                const cudaError_t e = cudaFuncSetAttribute(
-                    k, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kStageBytes));
-                if (e != cudaSuccess) attr_err = e;
-            }
-        });
+        const cudaError_t attr_err = func_attr_once(reinterpret_cast<const void *>(kern),
+                                                    cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                    static_cast<int>(kStageBytes));
         if (attr_err != cudaSuccess) return attr_err;
         return launch_pdl(kern, grid, dim3(kThreads), kStageBytes, s, a, TB, l_per_cta);
     } else {

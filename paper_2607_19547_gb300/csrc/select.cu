@@ -193,6 +193,12 @@ select_kernel(const uint32_t *__restrict__ score, int n, int k, int idx_base, in
 
     for (int j = t; j < 2 * kBins; j += kNT) (&s->hist[0][0])[j] = 0u;
     if (t < 2 * kGroups) (&s->coarse[0][0])[t] = 0u;
+    if (t == 0) {   // defined even if a search found nothing (the counts rule that out)
+        s->s_group = 0;
+        s->s_above = 0;
+        s->s_hit = 0;
+        s->s_cnt = 0;
+    }
     __syncthreads();
 
     // a word of this CTA's shared memory as seen in CTA c of the cluster (c == r: itself)
