@@ -26,7 +26,7 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int kMaxTokensPerCta = 32;   // fp32 kernel
-constexpr int kMaxTokensBf16 = 8;      // bf16 kernel: token block of 8 / n_kv_heads
+constexpr int kMaxTokensBf16 = 16;     // bf16 kernel: token block of 16 / n_kv_heads
 constexpr int kMaxBlocks = 512;        // 8-element blocks of one token row (32 kv heads)
 
 // 1/n! split exactly into fp32 hi + lo (hi = fp32(1/n!), lo = fp32(1/n! - hi)).
@@ -150,8 +150,10 @@ __device__ __forceinline__ uint32_t pack_bf16x2_rn(float lo, float hi) {
 // only its own slots, so the copies need no block barrier: a wait on the thread's own
 // copy groups makes them visible to it.  Slot (stage s, half h) of thread x sits at
 // word (s * 2 + h) * kThreads + x, so a warp's reads and copies touch consecutive
-// 16-byte words.
-constexpr int kStages = 4;
+// 16-byte words.  Six stages (48 KB) with the cos/sin table beside them leave room
+// for three CTAs per SM; measured on the 3B shapes against four stages at four CTAs
+// per SM, and against three, five and eight stages, six was the fastest at every size.
+constexpr int kStages = 6;
 constexpr size_t kStageBytes = static_cast<size_t>(kStages) * 2 * kThreads * 16;
 
 __device__ __forceinline__ uint4 *stage_slot(uint4 *buf, int s, int h) {
@@ -410,15 +412,19 @@ __device__ __forceinline__ void stream_slices(const __nv_bfloat16 *src, __nv_bfl
 //     8 blocks stays inside a thread (its two halves), and 4, 2, 1 are lane
 //     offsets again.
 // HKV > 0: the kv head count is that compile-time constant (the token block is
-// then 8 / HKV tokens, 64 threads per layer slot, and the index arithmetic below
-// is shifts); HKV == 0: any head count, TB as passed.
+// then 16 / HKV tokens, 128 threads per layer slot, two slots, and the index
+// arithmetic below is shifts); HKV == 0: any head count, TB as passed.  Two slots
+// (each thread walks half of the CTA's layers) measured faster than four at every
+// size: half as many CTA prologues, and longer per-thread streams.
+// Dynamic shared memory: the kStages staging buffers, then the table (TB * 64 entries).
 template <int HKV>
-__global__ void __launch_bounds__(kThreads, 4) rebase_bf16_kernel(RebaseArgs a, int TB_arg, int l_per_cta) {
+__global__ void __launch_bounds__(kThreads, 3) rebase_bf16_kernel(RebaseArgs a, int TB_arg, int l_per_cta) {
     pdl_wait();   // inputs may come from the previous kernel of the stream
     pdl_trigger();
     const int hkv = HKV > 0 ? HKV : a.hkv;
-    const int TB = HKV > 0 ? 8 / HKV : TB_arg;
-    __shared__ float4 tab[kMaxTokensBf16 * 64];
+    const int TB = HKV > 0 ? 16 / HKV : TB_arg;
+    extern __shared__ uint4 stage[];
+    float4 *tab = reinterpret_cast<float4 *>(stage + kStages * 2 * kThreads);
     __shared__ int s_delta[kMaxTokensBf16][3];
     const int t0 = blockIdx.x * TB;
     const int l0 = blockIdx.y * l_per_cta;
@@ -447,7 +453,6 @@ __global__ void __launch_bounds__(kThreads, 4) rebase_bf16_kernel(RebaseArgs a, 
     const long long lstep = static_cast<long long>(n_slots) * a.layer_stride;
     const long long obase = static_cast<long long>(lfirst) * a.layer_stride + row0;
     // the first layers' words go out before the table is built (empty groups past count)
-    extern __shared__ uint4 stage[];
     for (int st = 0; st < kStages; ++st) {
         if (st < count) {
             cp_async16(stage_slot(stage, st, 0), src + obase + st * lstep);
@@ -617,8 +622,8 @@ bool rebase_fuses_score(const RebaseArgs &a, cs_dtype dt) {
 cudaError_t launch_rebase(const RebaseArgs &a, cs_dtype dt, cudaStream_t s) {
     if (a.T == 0 || a.n_layers == 0) return cudaSuccess;
     if (dt == CS_DTYPE_BF16) {
-        // token block: 64 threads per layer slot where possible (4 slots per CTA)
-        const int TB = a.hkv >= 8 ? 1 : 8 / a.hkv;
+        // token block: 128 threads per layer slot where possible (2 slots per CTA)
+        const int TB = a.hkv >= kMaxTokensBf16 ? 1 : kMaxTokensBf16 / a.hkv;
         const int blocks = (a.T + TB - 1) / TB;
         const int slots = kThreads / (TB * a.hkv * 8);
         // split layers across CTAs only when there are too few token blocks to fill
@@ -630,13 +635,16 @@ cudaError_t launch_rebase(const RebaseArgs &a, cs_dtype dt, cudaStream_t s) {
                                                (a.n_layers + slots - 1) / slots);
         const int l_per_cta = (a.n_layers + groups - 1) / groups;
         dim3 grid(blocks, (a.n_layers + l_per_cta - 1) / l_per_cta);
+        const size_t smem = kStageBytes + static_cast<size_t>(TB) * 64 * sizeof(float4);
         auto *kern = a.hkv == 1 ? rebase_bf16_kernel<1> : a.hkv == 2 ? rebase_bf16_kernel<2>
                    : a.hkv == 4 ? rebase_bf16_kernel<4> : rebase_bf16_kernel<0>;
+        // the limit covers the largest table, so one setting serves every head count
+        constexpr size_t kSmemMax = kStageBytes + kMaxTokensBf16 * 64 * sizeof(float4);
         const cudaError_t attr_err = func_attr_once(reinterpret_cast<const void *>(kern),
                                                     cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                    static_cast<int>(kStageBytes));
+                                                    static_cast<int>(kSmemMax));
         if (attr_err != cudaSuccess) return attr_err;
-        return launch_pdl(kern, grid, dim3(kThreads), kStageBytes, s, a, TB, l_per_cta);
+        return launch_pdl(kern, grid, dim3(kThreads), smem, s, a, TB, l_per_cta);
     } else {
         const int TB = a.hkv >= kMaxTokensPerCta / 2 ? 1 : (kMaxTokensPerCta / 2) / a.hkv;
         const int layers_per_cta = 4;
