@@ -2,8 +2,9 @@
 //
 // Scores map to order-preserving 32-bit keys; the k largest keys win, equal keys
 // rank the lower index first, and the output is the selected indices in
-// ascending order.  Exact radix select over one thread-block cluster of C CTAs
-// (C = 1, 2, 4, 8 or 16, sized from n):
+// ascending order.  Up to 4096 scores: one CTA (select_small_kernel below).  Beyond
+// that: exact radix select over one thread-block cluster of C CTAs (C = 2, 4, 8 or 16,
+// sized from n; 1 where the device cannot co-schedule a cluster):
 //   - CTA r owns the contiguous candidate range [r*span, (r+1)*span) and thread t
 //     of it the contiguous range [t*per, (t+1)*per) inside that; up to 16 keys per
 //     thread stay in registers (16-byte loads), larger inputs are re-read in every
@@ -332,6 +333,201 @@ select_kernel(const uint32_t *__restrict__ score, int n, int k, int idx_base, in
     if (C > 1) cluster_wait();   // others may still read this CTA's counts until here
 }
 
+// ---- one CTA, up to kSmallN keys -------------------------------------------------
+//
+// For small inputs the cluster machinery costs more than the counting, so one CTA of
+// kNT threads (eight keys each, in registers) runs a leaner form of the same exact
+// selection:
+//   - the digits start at the highest bit in which the smallest and largest key differ
+//     (every key shares the bits above it), so the first 11-bit digit already splits
+//     the populated key range;
+//   - after each histogram one warp finds the bin of the k-th largest key: lane l sums
+//     the 64 bins [2048 - 64(l+1), 2048 - 64 l) (lane 0 the highest), a warp scan picks
+//     the lane, a second scan over that lane's bins (two per lane) picks the bin; the
+//     rest of the CTA waits at one barrier;
+//   - when that bin holds at most kCand keys and not all of them are taken, its keys are
+//     gathered in shared memory and one warp ranks them directly (each candidate counts
+//     the candidates above it), which gives K* without further passes;
+//   - the final counts (greater, equal) fit in 16 bits each, so one 32-bit block scan
+//     gives every thread its first output position.
+constexpr int kSmallN = kNT * 8;
+constexpr int kCand = 64;
+
+struct SmallShared {
+    uint32_t hist[2][kBins];            // double-buffered: a pass clears the one it read
+    uint32_t wmin[kWarps], wmax[kWarps];
+    uint32_t wsum[kWarps];
+    uint32_t cand[kCand];
+    uint32_t s_hit, s_above, s_cnt, s_ncand, s_kstar, s_krem;
+};
+
+// Warp 0 only: the bin of hist (kBins bins, digit order) that holds the krem-th largest
+// key, the keys above it and its count, into s_hit / s_above / s_cnt.  The histogram
+// holds at least krem keys.
+__device__ __forceinline__ void small_find_bin(const uint32_t *hist, uint32_t krem,
+                                               SmallShared *s) {
+    const int lane = threadIdx.x & 31;
+    const uint4 *h4 = reinterpret_cast<const uint4 *>(hist) + (kBins - 64 * (lane + 1)) / 4;
+    uint32_t sum = 0;
+#pragma unroll
+    for (int q = 0; q < 16; ++q) {   // rotated start: the lanes of a phase hit distinct banks
+        const uint4 v = h4[(q + lane) & 15];
+        sum += v.x + v.y + v.z + v.w;
+    }
+    const uint32_t incl = warp_incl_scan(sum);
+    const uint32_t above = incl - sum;
+    const int L = __ffs(__ballot_sync(0xFFFFFFFFu, above < krem && incl >= krem)) - 1;
+    const uint32_t above_l = __shfl_sync(0xFFFFFFFFu, above, L);
+    // lane j: bins b and b - 1 of lane L's chunk, b = its top bin - 2j (descending)
+    const int b = kBins - 64 * L - 1 - 2 * lane;
+    const uint32_t f1 = hist[b], f2 = hist[b - 1];
+    const uint32_t incl2 = warp_incl_scan(f1 + f2);
+    const uint32_t above2 = incl2 - f1 - f2, want = krem - above_l;
+    if (above2 < want && incl2 >= want) {
+        const bool top = above2 + f1 >= want;
+        s->s_hit = static_cast<uint32_t>(top ? b : b - 1);
+        s->s_above = above_l + (top ? above2 : above2 + f1);
+        s->s_cnt = top ? f1 : f2;
+    }
+}
+
+__global__ void __launch_bounds__(kNT, 1)
+select_small_kernel(const uint32_t *__restrict__ score, int n, int k, int idx_base, int vec,
+                    int *__restrict__ out) {
+    pdl_wait();   // inputs may come from the previous kernel of the stream
+    pdl_trigger();
+    __shared__ __align__(16) SmallShared sh;
+    SmallShared *s = &sh;
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const int i0 = t * 8;
+    const int cnt = max(0, min(8, n - i0));
+    if (k >= n) {   // everything is selected, in index order (no barrier on this path)
+        for (int i = 0; i < cnt; ++i) out[i0 + i] = idx_base + i0 + i;
+        return;
+    }
+    uint32_t reg[8];
+    if (vec && cnt == 8) {
+        const uint4 u = __ldg(reinterpret_cast<const uint4 *>(score + i0));
+        const uint4 v = __ldg(reinterpret_cast<const uint4 *>(score + i0 + 4));
+        reg[0] = order_key(u.x); reg[1] = order_key(u.y); reg[2] = order_key(u.z); reg[3] = order_key(u.w);
+        reg[4] = order_key(v.x); reg[5] = order_key(v.y); reg[6] = order_key(v.z); reg[7] = order_key(v.w);
+    } else {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) reg[i] = i < cnt ? order_key(__ldg(score + i0 + i)) : 0u;
+    }
+    uint32_t lo = 0xFFFFFFFFu, hi = 0u;
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+        if (i < cnt) {
+            lo = min(lo, reg[i]);
+            hi = max(hi, reg[i]);
+        }
+    lo = __reduce_min_sync(0xFFFFFFFFu, lo);
+    hi = __reduce_max_sync(0xFFFFFFFFu, hi);
+    if (lane == 0) {
+        s->wmin[warp] = lo;
+        s->wmax[warp] = hi;
+    }
+    {
+        uint4 *h = reinterpret_cast<uint4 *>(&s->hist[0][0]);
+        for (int j = t; j < 2 * kBins / 4; j += kNT) h[j] = make_uint4(0, 0, 0, 0);
+    }
+    if (t == 0) {
+        s->s_ncand = 0;
+        s->s_hit = 0;
+        s->s_above = 0;
+        s->s_cnt = 0;
+        s->s_kstar = 0;
+        s->s_krem = 0;
+    }
+    __syncthreads();
+    const uint32_t kmin = __reduce_min_sync(0xFFFFFFFFu, s->wmin[lane % kWarps]);
+    const uint32_t kmax = __reduce_max_sync(0xFFFFFFFFu, s->wmax[lane % kWarps]);
+
+    // prefix = the resolved high bits of K*, pmask their mask; krem = how many keys with
+    // that prefix are still to be selected; nxt = the number of unresolved low bits
+    const uint32_t diff = kmin ^ kmax;
+    int nxt = diff ? 32 - __clz(diff) : 0;
+    uint32_t pmask = nxt == 32 ? 0u : ~((1u << nxt) - 1u);
+    uint32_t prefix = kmax & pmask;
+    uint32_t krem = static_cast<uint32_t>(k);
+    int buf = 0;
+#pragma unroll 1
+    while (nxt > 0) {
+        const int shift = max(nxt - 11, 0);
+        const uint32_t dmask = (1u << (nxt - shift)) - 1u;
+        uint32_t *hist = s->hist[buf];
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+            if (i < cnt && (reg[i] & pmask) == prefix) atomicAdd(&hist[(reg[i] >> shift) & dmask], 1u);
+        __syncthreads();
+        if (warp == 0) small_find_bin(hist, krem, s);
+        __syncthreads();
+        const uint32_t c_bin = s->s_cnt;
+        prefix |= s->s_hit << shift;
+        pmask |= dmask << shift;
+        krem -= s->s_above;
+        nxt = shift;
+        // every key left in the bin is taken, or the bin is one key value: K* is resolved
+        // as far as the selection needs
+        if (c_bin == krem || nxt == 0) break;
+        if (c_bin <= static_cast<uint32_t>(kCand)) {
+            // rank the bin's keys directly
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+                if (i < cnt && (reg[i] & pmask) == prefix) s->cand[atomicAdd(&s->s_ncand, 1u)] = reg[i];
+            __syncthreads();
+            if (warp == 0) {
+                for (int j = lane; j < static_cast<int>(c_bin); j += 32) {
+                    const uint32_t x = s->cand[j];
+                    uint32_t gt = 0, ge = 0;
+                    for (int q = 0; q < static_cast<int>(c_bin); ++q) {
+                        const uint32_t y = s->cand[q];
+                        gt += y > x;
+                        ge += y >= x;
+                    }
+                    if (gt < krem && ge >= krem) {   // x is K* (equal candidates agree)
+                        s->s_kstar = x;
+                        s->s_krem = krem - gt;
+                    }
+                }
+            }
+            __syncthreads();
+            prefix = s->s_kstar;
+            pmask = 0xFFFFFFFFu;
+            krem = s->s_krem;
+            break;
+        }
+        // another histogram pass over the next digit: clear the buffer just read (the
+        // pass after next uses it; a barrier separates the two)
+        for (int j = t; j < kBins / 4; j += kNT)
+            reinterpret_cast<uint4 *>(hist)[j] = make_uint4(0, 0, 0, 0);
+        buf ^= 1;
+    }
+
+    // K* = prefix under pmask; keys above it are taken, and the first krem equal to it
+    const uint32_t kstar = prefix;
+    uint32_t gt = 0, eq = 0;
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+        if (i < cnt) {
+            const uint32_t km = reg[i] & pmask;
+            gt += km > kstar;
+            eq += km == kstar;
+        }
+    // both counts stay below 2^16 over the whole CTA (n <= kSmallN)
+    const uint32_t mine = (gt << 16) | eq;
+    const uint32_t before = block_incl_scan<uint32_t>(mine, s->wsum) - mine;
+    uint32_t eq_seen = before & 0xFFFFu;
+    uint32_t pos = (before >> 16) + min(eq_seen, krem);
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+        if (i < cnt) {
+            const uint32_t km = reg[i] & pmask;
+            if (km > kstar || (km == kstar && eq_seen++ < krem)) out[pos++] = idx_base + i0 + i;
+        }
+}
+
 // The largest cluster size (a power of two <= 16) the device can co-schedule for
 // kernel number `which` (0..3); cached per kernel and device.
 int max_cluster(int which, void (*kernel)(const uint32_t *, int, int, int, int, int, int *)) {
@@ -402,6 +598,18 @@ cudaError_t launch_select(const float *score, int n, int k, int idx_base, int *o
     if (k == 0 || n == 0) return cudaSuccess;
     const uint32_t *keys = reinterpret_cast<const uint32_t *>(score);
     const int vec = (reinterpret_cast<uintptr_t>(score) & 15u) == 0;
+    if (n <= kSmallN) {
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(1);
+        cfg.blockDim = dim3(kNT);
+        cfg.stream = s;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        return cudaLaunchKernelEx(&cfg, select_small_kernel, keys, n, k, idx_base, vec, out);
+    }
     // cluster size: about 4096 keys per CTA, a power of two up to what the device allows
     int want = 1;
     while (want < kMaxCluster && static_cast<long long>(want) * 4096 < n) want *= 2;

@@ -120,3 +120,28 @@ def test_select_ties_across_ctas(cslib):
     vals[::1000] = 9.0
     for k in (1, 65, 30000, n - 3):
         _check_select(cslib, vals, k, 1032)
+
+
+@pytest.mark.parametrize("n", [2, 100, 3000, 4096])
+def test_select_small_input_paths(cslib, n):
+    """Inputs of one CTA (up to 4096 scores): a key range spanning all 32 bits, a tight
+    cluster that needs three digit passes (the keys differ only in their 12 lowest bits
+    below two outliers), a range of a few low bits only, signed values, and scores that
+    start 4 bytes past a 16-byte boundary."""
+    rng = np.random.default_rng(7 * n)
+    wide = (rng.lognormal(0, 3, n) * rng.choice([-1.0, 1.0], n)).astype(np.float32)
+    bits = (np.float32(1.0).view(np.uint32) + rng.integers(0, 4096, n)).astype(np.uint32)
+    cluster = bits.view(np.float32).copy()
+    cluster[0], cluster[-1] = 1e30, 0.0
+    narrow = (np.float32(3.0).view(np.uint32) + rng.integers(0, 8, n)).astype(np.uint32)
+    narrow = narrow.view(np.float32)
+    for vals in (wide, cluster, narrow):
+        for k in sorted({1, max(n // 10, 1), n // 2, max(n - 1, 1)}):
+            _check_select(cslib, vals, k, 5)
+    buf = cuda(np.concatenate([[np.float32(9.0)], wide]).astype(np.float32))
+    view = buf[1:]
+    assert view.data_ptr() % 16 == 4
+    for k in sorted({1, max(n // 3, 1), max(n - 1, 1)}):
+        got = cslib.cs_select_topk(view, k, 0).cpu().numpy()
+        cslib.cs_sync_status()
+        assert np.array_equal(got, O.select_topk(wide, k, 0))
