@@ -2,7 +2,7 @@
 //
 // Scores map to order-preserving 32-bit keys; the k largest keys win, equal keys
 // rank the lower index first, and the output is the selected indices in
-// ascending order.  Up to 4096 scores: one CTA (select_small_kernel below).  Beyond
+// ascending order.  Up to 8192 scores: one CTA (select_small_kernel below).  Beyond
 // that: exact radix select over one thread-block cluster of C CTAs (C = 2, 4, 8 or 16,
 // sized from n; 1 where the device cannot co-schedule a cluster):
 //   - CTA r owns the contiguous candidate range [r*span, (r+1)*span) and thread t
@@ -336,7 +336,7 @@ select_kernel(const uint32_t *__restrict__ score, int n, int k, int idx_base, in
 // ---- one CTA, up to kSmallN keys -------------------------------------------------
 //
 // For small inputs the cluster machinery costs more than the counting, so one CTA of
-// kNT threads (eight keys each, in registers) runs a leaner form of the same exact
+// kNT threads (8 or 16 keys each, in registers) runs a leaner form of the same exact
 // selection:
 //   - the digits start at the highest bit in which the smallest and largest key differ
 //     (every key shares the bits above it), so the first 11-bit digit already splits
@@ -350,7 +350,7 @@ select_kernel(const uint32_t *__restrict__ score, int n, int k, int idx_base, in
 //     the candidates above it), which gives K* without further passes;
 //   - the final counts (greater, equal) fit in 16 bits each, so one 32-bit block scan
 //     gives every thread its first output position.
-constexpr int kSmallN = kNT * 8;
+constexpr int kSmallN = kNT * 16;
 constexpr int kCand = 64;
 
 struct SmallShared {
@@ -391,6 +391,7 @@ __device__ __forceinline__ void small_find_bin(const uint32_t *hist, uint32_t kr
     }
 }
 
+template <int KPT>
 __global__ void __launch_bounds__(kNT, 1)
 select_small_kernel(const uint32_t *__restrict__ score, int n, int k, int idx_base, int vec,
                     int *__restrict__ out) {
@@ -399,25 +400,29 @@ select_small_kernel(const uint32_t *__restrict__ score, int n, int k, int idx_ba
     __shared__ __align__(16) SmallShared sh;
     SmallShared *s = &sh;
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
-    const int i0 = t * 8;
-    const int cnt = max(0, min(8, n - i0));
+    const int i0 = t * KPT;
+    const int cnt = max(0, min(KPT, n - i0));
     if (k >= n) {   // everything is selected, in index order (no barrier on this path)
         for (int i = 0; i < cnt; ++i) out[i0 + i] = idx_base + i0 + i;
         return;
     }
-    uint32_t reg[8];
-    if (vec && cnt == 8) {
-        const uint4 u = __ldg(reinterpret_cast<const uint4 *>(score + i0));
-        const uint4 v = __ldg(reinterpret_cast<const uint4 *>(score + i0 + 4));
-        reg[0] = order_key(u.x); reg[1] = order_key(u.y); reg[2] = order_key(u.z); reg[3] = order_key(u.w);
-        reg[4] = order_key(v.x); reg[5] = order_key(v.y); reg[6] = order_key(v.z); reg[7] = order_key(v.w);
+    uint32_t reg[KPT];
+    if (vec && cnt == KPT) {
+#pragma unroll
+        for (int c = 0; c < KPT / 4; ++c) {
+            const uint4 u = __ldg(reinterpret_cast<const uint4 *>(score + i0) + c);
+            reg[4 * c] = order_key(u.x);
+            reg[4 * c + 1] = order_key(u.y);
+            reg[4 * c + 2] = order_key(u.z);
+            reg[4 * c + 3] = order_key(u.w);
+        }
     } else {
 #pragma unroll
-        for (int i = 0; i < 8; ++i) reg[i] = i < cnt ? order_key(__ldg(score + i0 + i)) : 0u;
+        for (int i = 0; i < KPT; ++i) reg[i] = i < cnt ? order_key(__ldg(score + i0 + i)) : 0u;
     }
     uint32_t lo = 0xFFFFFFFFu, hi = 0u;
 #pragma unroll
-    for (int i = 0; i < 8; ++i)
+    for (int i = 0; i < KPT; ++i)
         if (i < cnt) {
             lo = min(lo, reg[i]);
             hi = max(hi, reg[i]);
@@ -458,7 +463,7 @@ select_small_kernel(const uint32_t *__restrict__ score, int n, int k, int idx_ba
         const uint32_t dmask = (1u << (nxt - shift)) - 1u;
         uint32_t *hist = s->hist[buf];
 #pragma unroll
-        for (int i = 0; i < 8; ++i)
+        for (int i = 0; i < KPT; ++i)
             if (i < cnt && (reg[i] & pmask) == prefix) atomicAdd(&hist[(reg[i] >> shift) & dmask], 1u);
         __syncthreads();
         if (warp == 0) small_find_bin(hist, krem, s);
@@ -474,7 +479,7 @@ select_small_kernel(const uint32_t *__restrict__ score, int n, int k, int idx_ba
         if (c_bin <= static_cast<uint32_t>(kCand)) {
             // rank the bin's keys directly
 #pragma unroll
-            for (int i = 0; i < 8; ++i)
+            for (int i = 0; i < KPT; ++i)
                 if (i < cnt && (reg[i] & pmask) == prefix) s->cand[atomicAdd(&s->s_ncand, 1u)] = reg[i];
             __syncthreads();
             if (warp == 0) {
@@ -509,7 +514,7 @@ select_small_kernel(const uint32_t *__restrict__ score, int n, int k, int idx_ba
     const uint32_t kstar = prefix;
     uint32_t gt = 0, eq = 0;
 #pragma unroll
-    for (int i = 0; i < 8; ++i)
+    for (int i = 0; i < KPT; ++i)
         if (i < cnt) {
             const uint32_t km = reg[i] & pmask;
             gt += km > kstar;
@@ -521,7 +526,7 @@ select_small_kernel(const uint32_t *__restrict__ score, int n, int k, int idx_ba
     uint32_t eq_seen = before & 0xFFFFu;
     uint32_t pos = (before >> 16) + min(eq_seen, krem);
 #pragma unroll
-    for (int i = 0; i < 8; ++i)
+    for (int i = 0; i < KPT; ++i)
         if (i < cnt) {
             const uint32_t km = reg[i] & pmask;
             if (km > kstar || (km == kstar && eq_seen++ < krem)) out[pos++] = idx_base + i0 + i;
@@ -608,7 +613,9 @@ cudaError_t launch_select(const float *score, int n, int k, int idx_base, int *o
         attr[0].val.programmaticStreamSerializationAllowed = 1;
         cfg.attrs = attr;
         cfg.numAttrs = 1;
-        return cudaLaunchKernelEx(&cfg, select_small_kernel, keys, n, k, idx_base, vec, out);
+        if (n <= kNT * 8)
+            return cudaLaunchKernelEx(&cfg, select_small_kernel<8>, keys, n, k, idx_base, vec, out);
+        return cudaLaunchKernelEx(&cfg, select_small_kernel<16>, keys, n, k, idx_base, vec, out);
     }
     // cluster size: about 4096 keys per CTA, a power of two up to what the device allows
     int want = 1;

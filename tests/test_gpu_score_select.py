@@ -122,9 +122,9 @@ def test_select_ties_across_ctas(cslib):
         _check_select(cslib, vals, k, 1032)
 
 
-@pytest.mark.parametrize("n", [2, 100, 3000, 4096])
+@pytest.mark.parametrize("n", [2, 100, 3000, 4096, 6000, 8192])
 def test_select_small_input_paths(cslib, n):
-    """Inputs of one CTA (up to 4096 scores): a key range spanning all 32 bits, a tight
+    """Inputs of one CTA (up to 8 192 scores): a key range spanning all 32 bits, a tight
     cluster that needs three digit passes (the keys differ only in their 12 lowest bits
     below two outliers), a range of a few low bits only, signed values, and scores that
     start 4 bytes past a 16-byte boundary."""
