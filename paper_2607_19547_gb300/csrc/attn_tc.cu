@@ -31,8 +31,11 @@
 //               The running max is raised only when it grows by more than
 //               2^8; when that happens in either half, both warps exchange
 //               their maxima through shared memory, raise it, recompute P_j
-//               from S_j and rescale their half of O in TMEM.  P_j is written
-//               as bf16 over S_j's TMEM columns.  Finally each warp normalises
+//               from S_j and rescale their half of O in TMEM.  Each warp writes
+//               its half of P_j as bf16 over the first 32 of its own 64 S_j
+//               columns (never over columns the other warp reads), and the P*V
+//               issuer takes keys [64h, 64h+64) from columns [64h, 64h+32).
+//               Finally each warp normalises
 //               its half of O into the Q tile's shared memory (idle after the
 //               last S), from where two TMA stores write whole rows.
 // TMEM: S buffers at columns 0, 128, 256; O at 384.  S_j reuses the buffer
@@ -318,9 +321,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
                 const uint32_t a_tm = tmem + static_cast<uint32_t>(b * kBlockN);
 #pragma unroll
                 for (int kk = 0; kk < kBlockN / 16; ++kk) {
-                    // A: 16 keys of P = 8 packed columns; B: 16 rows (keys) of V, MN-major
-                    tc_mma_ts(tmem + kColO, a_tm + kk * 8, vd + ((kk * 2048) >> 4), idesc,
-                              (j > 0 || kk > 0) ? 1u : 0u);
+                    // A: 16 keys of P = 8 packed columns (keys [64h, 64h+64) sit in columns
+                    // [64h, 64h+32) of the buffer); B: 16 rows (keys) of V, MN-major
+                    tc_mma_ts(tmem + kColO, a_tm + (kk >> 2) * 64 + (kk & 3) * 8,
+                              vd + ((kk * 2048) >> 4), idesc, (j > 0 || kk > 0) ? 1u : 0u);
                 }
                 tc_commit(&bars->pv_done[b]);
                 tc_commit(&bars->v_empty[s]);
@@ -412,8 +416,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
                 load_s_half(s_addr, diag, lim, s);
                 psum = exp_pack(s, p.scale_log2, m_run, pk);
             }
-            // packed bf16 into columns [32h, 32h+32) of S_j's buffer
-            tmem_st32(lane_base + b * kBlockN + 32 * half, pk);
+            // packed bf16 into columns [64h, 64h+32) of S_j's buffer: inside this warp's
+            // own half of S_j, which it has read already, so no other warp's read of S_j can
+            // meet this store
+            tmem_st32(lane_base + b * kBlockN + col0, pk);
             l_run += psum;
             // rescale this half of O when any row of the warp raised its max
             // (O holds PV_0 .. PV_{j-1})
