@@ -154,9 +154,9 @@ cs_status cs_rebase_and_score(const void *k_in, void *k_out, cs_dtype dtype, int
  *
  *   score    fp32 [n], device memory;   0 <= k <= n;   idx_base + n <= INT32_MAX
  *   out_idx  int32 [k], device memory, not overlapping score (CS_ERR_INVALID_ARG)
- * One launch of one thread-block cluster (up to 16 CTAs, as many as the device can
- * co-schedule; the first call on a device queries that, so make it before capturing a
- * stream); no global memory besides score and out_idx is used.
+ * One launch: one CTA for n <= 8192, else one thread-block cluster (up to 16 CTAs, as
+ * many as the device can co-schedule; the first such call on a device queries that, so
+ * make it before capturing a stream); no global memory besides score and out_idx is used.
  */
 cs_status cs_select_topk(const float *score, int n, int k, int32_t idx_base, int32_t *out_idx,
                          void *stream);
