@@ -44,6 +44,19 @@ def test_tiny_f32_config_full(cslib):
     _run_and_check(cslib, x["q"], x["k"], x["v"], qpos, "f32")
 
 
+@pytest.mark.parametrize("Hq,Hkv", [(2, 1), (8, 2), (6, 3)])
+def test_f32_key_chunks_ragged(cslib, Hq, Hkv):
+    """fp32 path: rows whose visible keys end on, before and after the 32-key chunk edges,
+    including the first key alone, over two layers."""
+    L, T = 2, 300
+    qpos = np.array([0, 1, 30, 31, 32, 33, 63, 64, 65, 100, 127, 128, 200, 299], np.int32)
+    M = len(qpos)
+    q = _rand((L, M, Hq, 128), 21, torch.float32)
+    k = _rand((L, T, Hkv, 128), 22, torch.float32)
+    v = _rand((L, T, Hkv, 128), 23, torch.float32)
+    _run_and_check(cslib, q, k, v, qpos, "f32")
+
+
 @pytest.mark.parametrize("Hq,Hkv", [(16, 2), (28, 4), (2, 1), (8, 8), (7, 1), (32, 2)])
 def test_bf16_group_sizes_ragged(cslib, Hq, Hkv):
     L, T, M = 2, 1000, 37
