@@ -209,6 +209,77 @@ def config_of(w, ws: int) -> dict:
 
 # ----------------------------------------------------------------------------- GPU arm
 
+def _event_mean_ms(run, flush_l2, stream, reps: int) -> float:
+    """Mean device time of run() over reps calls, L2 flushed (untimed) before each."""
+    ms = []
+    for _ in range(reps):
+        flush_l2()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        run()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms.append(e0.elapsed_time(e1))
+    return float(np.mean(ms))
+
+
+def measure_next_rows(w, x, q, flush_l2, stream, pk, reps: int = 5) -> dict:
+    """The two next-step kernels of the query outside the timed step, on the same workload:
+
+    * scatter-back (Sec. 2): fresh K and V rows of the k repaired tokens, all layers, written
+      into the cache at the step's selected positions (two cs_scatter_rows calls); bytes =
+      the fresh rows read + the cache rows written, for K and V;
+    * shallow recompute (Eq. 6, 2 c_a |C| T): every candidate as a query row over the first
+      two layers (cs_repair_attention through ComposedQuery.shallow_recompute); FLOP as for
+      the repair attention over the candidates' positions.
+
+    Inputs are seeded random draws of the right shapes; V's overwritten rows are restored
+    afterwards (K is restored by every step)."""
+    import paper_2607_19547_gb300 as cs
+
+    dev = x["k"].device
+    g = torch.Generator(device=dev).manual_seed(20260)
+    L, k, b = w.n_layers, w.k, w.elem_bytes
+    idx = q.qpos[:k]
+    rows = lambda: torch.randn((L, k, w.hkv, w.head_dim), generator=g, device=dev).to(w.torch_dtype)  # noqa: E731
+    k_rows, v_rows = rows(), rows()
+    v_saved = x["v"][:, idx.long()].clone()
+
+    def scatter():
+        cs.cs_scatter_rows(x["k"], k_rows, idx)
+        cs.cs_scatter_rows(x["v"], v_rows, idx)
+
+    scatter()
+    torch.cuda.synchronize()
+    sc_ms = _event_mean_ms(scatter, flush_l2, stream, reps)
+    x["v"][:, idx.long()] = v_saved
+    sc_bytes = 2.0 * 2.0 * L * k * w.hkv * w.head_dim * b + 2.0 * 4.0 * k
+    sc_gbs = sc_bytes / (sc_ms / 1e3) / 1e9
+    out = {"scatter_back": {"us": round(sc_ms * 1e3, 2), "bytes": sc_bytes,
+                            "gbs": round(sc_gbs, 1), "frac_hbm": round(sc_gbs / pk["hbm_gbs"], 4),
+                            "launches": 2, "rows": f"{L} layers x {k} rows, K and V",
+                            "timed": f"event around the two calls, mean of {reps}, L2 flushed"}}
+    nl = min(2, L)
+    q_cand = torch.randn((nl, w.n_cand, w.hq, w.head_dim), generator=g, device=dev).to(w.torch_dtype)
+    o_cand = torch.empty_like(q_cand)
+    run = lambda: q.shallow_recompute(q_cand, x["k"], x["v"], out=o_cand)   # noqa: E731
+    run()
+    torch.cuda.synchronize()
+    sr_reps = max(2, reps // 2)
+    sr_ms = _event_mean_ms(run, flush_l2, stream, sr_reps)
+    cs.cs_sync_status()
+    pos = np.arange(w.cand0, w.cand0 + w.n_cand, dtype=np.int64)
+    flop = 4.0 * w.head_dim * w.hq * nl * float(np.sum(pos + 1))
+    tflops = flop / (sr_ms / 1e3) / 1e12
+    out["shallow_recompute"] = {
+        "us": round(sr_ms * 1e3, 2), "flop": flop, "tflops": round(tflops, 2),
+        "frac_tensor": round(tflops / pk["bf16_tflops"], 4) if w.dtype == "bf16" else None,
+        "rows": f"{w.n_cand} candidates x {nl} layers",
+        "kernel": "attn_tc_kernel" if w.dtype == "bf16" else "attn_f32_kernel",
+        "timed": f"event around the call, mean of {sr_reps}, L2 flushed"}
+    return out
+
+
 def run_gpu(args, w, ws, rank, local):
     import paper_2607_19547_gb300 as cs
     from paper_2607_19547_gb300.pipeline import (ComposedQuery, GraphedQuery, PipelinedQuery,
@@ -352,6 +423,7 @@ def run_gpu(args, w, ws, rank, local):
     config = config_of(w, ws)
     if args.layers is not None:
         config["profiling_slice"] = f"first {w.n_layers} layers only (--layers)"
+    next_rows = None if args.no_next_rows else measure_next_rows(w, x, q, flush_l2, stream, pk)
 
     line = {
         "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": ws,
@@ -363,6 +435,8 @@ def run_gpu(args, w, ws, rank, local):
         "clocks": clk,
         "wall_s_timed_loop": round(wall, 4),
     }
+    if next_rows is not None:
+        line["next_rows"] = next_rows
     if args.no_e2e:
         return line, x, pristine
 
@@ -706,6 +780,8 @@ def main():
                     help="run re-base and score as two calls (the standalone score kernel), "
                          "not the fused cs_rebase_and_score launch")
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end (host buffer) leg")
+    ap.add_argument("--no-next-rows", action="store_true",
+                    help="skip the scatter-back and shallow-recompute measurements")
     ap.add_argument("--layers", type=int, default=None,
                     help="profiling aid: run only the first N layers of the workload (the line "
                          "says so; not a headline number)")
