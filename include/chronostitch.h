@@ -83,7 +83,8 @@ int cs_abi_version(void);
  *                 k_out == k_in re-bases in place (tokens with Delta = 0 are
  *                 not touched); otherwise every row of k_out is written and the
  *                 buffers must not overlap.
- *   pos_local, pos_global   int32 [T][3] (t, h, w) coordinates, device memory.
+ *   pos_local, pos_global   int32 [T][3] (t, h, w) coordinates, device memory,
+ *                 not overlapping k_out (CS_ERR_INVALID_ARG).
  *   rope          host pointer, read during the call only.
  *
  * Result: bf16 outputs are the exact rotation rounded once to bfloat16
@@ -131,7 +132,8 @@ cs_status cs_score_deviation(const void *k_fresh, const void *k_cached, cs_dtype
  *   0 <= score_layer < n_layers (when n_cand > 0);  0 <= cand0,  cand0 + n_cand <= T
  *   k_fresh    row c (token cand0 + c) at k_fresh + c*fresh_row_stride, E elements,
  *              device memory, 16-byte aligned rows, not overlapping k_out
- *   score_out  fp32 [n_cand], device memory, not overlapping the keys or k_fresh
+ *   score_out  fp32 [n_cand], device memory, not overlapping the keys, k_fresh or
+ *              the coordinates
  * Other arguments and errors as for cs_rebase_keys and cs_score_deviation.
  */
 cs_status cs_rebase_and_score(const void *k_in, void *k_out, cs_dtype dtype, int n_layers,
@@ -174,7 +176,7 @@ cs_status cs_select_topk(const float *score, int n, int k, int32_t idx_base, int
  *   k, v     [n_layers][T][n_kv_heads][head_dim] with layer stride kv_layer_stride
  *   qpos     int32 [M], strictly ascending, 0 <= qpos[r] < T (checked on the
  *            device; a violation yields CS_ERR_DEVICE_ARG at cs_sync_status and
- *            leaves o undefined)
+ *            leaves o undefined); not overlapping o or lse (CS_ERR_INVALID_ARG)
  *   lse      optional fp32 [n_layers][M][n_q_heads]: the natural-log normaliser
  *            log(sum_j exp(scale * q.k_j)); NULL to skip; 4-byte aligned and
  *            not overlapping k, v or o (CS_ERR_INVALID_ARG)
@@ -197,7 +199,8 @@ cs_status cs_repair_attention(const void *q, const void *k, const void *v, void 
  *              (elements, >= T*row_elems), device memory, written in place
  *   rows       [n_layers][n_rows][row_elems], layer stride rows_layer_stride
  *              (>= n_rows*row_elems), device memory, read only; must not overlap cache
- *   idx        int32 [n_rows], device memory, distinct destination tokens;
+ *   idx        int32 [n_rows], device memory, distinct destination tokens, not
+ *              overlapping cache (CS_ERR_INVALID_ARG);
  *              0 <= idx[r] < T is checked on the device: a row outside is
  *              skipped and cs_sync_status then returns CS_ERR_DEVICE_ARG
  *   row_elems  elements of one token row, e.g. n_kv_heads * head_dim; the row

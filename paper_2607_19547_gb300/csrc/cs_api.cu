@@ -118,6 +118,7 @@ cudaError_t func_attr_once(const void *fn, cudaFuncAttribute attr, int value) {
         const void *fn;
         int dev;
         int attr;
+        int value;
         cudaError_t err;
     };
     static std::mutex mu;
@@ -128,10 +129,11 @@ cudaError_t func_attr_once(const void *fn, cudaFuncAttribute attr, int value) {
     if (e != cudaSuccess) return e;
     std::lock_guard<std::mutex> lock(mu);
     for (int i = 0; i < n_done; ++i)
-        if (done[i].fn == fn && done[i].dev == dev && done[i].attr == static_cast<int>(attr))
+        if (done[i].fn == fn && done[i].dev == dev && done[i].attr == static_cast<int>(attr) &&
+            done[i].value == value)
             return done[i].err;
     e = cudaFuncSetAttribute(fn, attr, value);
-    if (n_done < 64) done[n_done++] = Entry{fn, dev, static_cast<int>(attr), e};
+    if (n_done < 64) done[n_done++] = Entry{fn, dev, static_cast<int>(attr), value, e};
     return e;
 }
 
@@ -237,12 +239,18 @@ cs_status rebase_impl(const void *k_in, void *k_out, cs_dtype dtype, int n_layer
         return fail(CS_ERR_INVALID_ARG, "NULL tensor pointer");
     if (!aligned16(k_in) || !aligned16(k_out) || (layer_stride * esz) % 16)
         return fail(CS_ERR_INVALID_ARG, "keys must be 16-byte aligned (pointers and layer stride)");
-    if (k_in != k_out) {
-        const long long span = ((n_layers - 1) * layer_stride + T * row) * esz;
-        const char *a = static_cast<const char *>(k_in);
-        const char *b = static_cast<const char *>(k_out);
-        if (a < b + span && b < a + span)
-            return fail(CS_ERR_INVALID_ARG, "k_in and k_out overlap without being equal");
+    const long long key_span = ((n_layers - 1) * layer_stride + T * row) * esz;
+    if (k_in != k_out && overlaps(k_in, key_span, k_out, key_span))
+        return fail(CS_ERR_INVALID_ARG, "k_in and k_out overlap without being equal");
+    {
+        // every CTA reads its tokens' coordinates while others write keys (and scores)
+        const long long pos_bytes = 12ll * T;
+        if (overlaps(pos_local, pos_bytes, k_out, key_span) ||
+            overlaps(pos_global, pos_bytes, k_out, key_span))
+            return fail(CS_ERR_INVALID_ARG, "coordinates overlap the re-based keys");
+        if (scoring && (overlaps(pos_local, pos_bytes, sc->score_out, 4ll * sc->n_cand) ||
+                        overlaps(pos_global, pos_bytes, sc->score_out, 4ll * sc->n_cand)))
+            return fail(CS_ERR_INVALID_ARG, "coordinates overlap score_out");
     }
     RebaseArgs args;
     std::memset(&args, 0, sizeof(args));
@@ -376,6 +384,9 @@ cs_status cs_scatter_rows(void *cache, const void *rows, cs_dtype dtype, int n_l
         const long long cspan = ((n_layers - 1) * cache_layer_stride + static_cast<long long>(T) * row_elems) * esz;
         const long long rspan = ((n_layers - 1) * rows_layer_stride + static_cast<long long>(n_rows) * row_elems) * esz;
         if (c < r + rspan && r < c + cspan) return fail(CS_ERR_INVALID_ARG, "rows overlap the cache");
+        // every warp reads its row's index while others write the cache
+        if (overlaps(idx, 4ll * n_rows, cache, cspan))
+            return fail(CS_ERR_INVALID_ARG, "idx overlaps the cache");
     }
     unsigned int *status = status_word();
     if (status == nullptr) return CS_ERR_CUDA;
@@ -434,7 +445,12 @@ cs_status cs_repair_attention(const void *q, const void *k, const void *v, void 
                 return fail(CS_ERR_INVALID_ARG, "lse overlaps k or v");
             if (lc < oc + o_span && oc < lc + l_span)
                 return fail(CS_ERR_INVALID_ARG, "lse overlaps o");
+            if (overlaps(qpos, 4ll * M, lse, l_span))
+                return fail(CS_ERR_INVALID_ARG, "qpos overlaps lse");
         }
+        // every CTA reads query positions while others write o (and lse)
+        if (overlaps(qpos, 4ll * M, o, o_span))
+            return fail(CS_ERR_INVALID_ARG, "qpos overlaps o");
     }
     unsigned int *status = status_word();
     if (status == nullptr) return CS_ERR_CUDA;

@@ -80,6 +80,12 @@ def test_rebase_rejects_bad_arguments(cslib):
     assert call(k_in=FAKE + 8, k_out=FAKE + 8) == cslib.CS_ERR_INVALID_ARG     # misaligned
     assert call(k_out=FAKE + 256) == cslib.CS_ERR_INVALID_ARG                  # partial overlap
     assert call(H=40) == cslib.CS_ERR_UNSUPPORTED
+    # coordinates are read while other CTAs write the keys
+    far = FAKE + (1 << 24)
+    assert call(pl=far, pg=FAKE + 512) == cslib.CS_ERR_INVALID_ARG
+    assert "coordinates overlap" in cslib.cs_last_error_detail()
+    assert call(pl=FAKE + 512, pg=far) == cslib.CS_ERR_INVALID_ARG
+    assert "coordinates overlap" in cslib.cs_last_error_detail()
     # nothing to do: succeeds without touching the device
     assert call(L=0, k_in=None, k_out=None) == cslib.CS_OK
     assert call(T=0, k_in=None, k_out=None, stride=0) == cslib.CS_OK
@@ -146,6 +152,11 @@ def test_attention_rejects_bad_arguments(cslib):
     assert "lse overlaps k or v" in cslib.cs_last_error_detail()
     assert call(o=far, lse=far + 256) == cslib.CS_ERR_INVALID_ARG
     assert "lse overlaps o" in cslib.cs_last_error_detail()
+    # query positions are read while other CTAs write o and lse
+    assert call(o=far, qpos=far + 64) == cslib.CS_ERR_INVALID_ARG
+    assert "qpos overlaps o" in cslib.cs_last_error_detail()
+    assert call(o=far, lse=far + (1 << 20), qpos=far + (1 << 20) + 8) == cslib.CS_ERR_INVALID_ARG
+    assert "qpos overlaps lse" in cslib.cs_last_error_detail()
 
 
 def test_debug_wait_rejects_bad_limits(cslib):
@@ -181,6 +192,8 @@ def test_scatter_rejects_bad_arguments(cslib):
     assert call(idx=None) == cslib.CS_ERR_INVALID_ARG
     assert call(cache=FAKE + 8) == cslib.CS_ERR_INVALID_ARG  # misaligned
     assert call(rows=FAKE + 512) == cslib.CS_ERR_INVALID_ARG  # overlaps the cache
+    assert call(idx=FAKE + 64) == cslib.CS_ERR_INVALID_ARG   # indices inside the cache
+    assert "idx overlaps" in cslib.cs_last_error_detail()
     assert call(T=0, cst=0) == cslib.CS_ERR_INVALID_ARG
     assert call(n=0, rows=None, idx=None) == cslib.CS_OK
     assert call(L=0) == cslib.CS_OK
@@ -210,4 +223,7 @@ def test_rebase_and_score_rejects_bad_arguments(cslib):
     assert "overlaps" in cslib.cs_last_error_detail()
     assert call(fr=FAKE + 256) == cslib.CS_ERR_INVALID_ARG  # fresh rows inside the keys
     assert "overlaps" in cslib.cs_last_error_detail()
+    far = FAKE + (1 << 26)
+    assert call(pl=far, pg=far, out=far + 64) == cslib.CS_ERR_INVALID_ARG
+    assert "coordinates overlap score_out" in cslib.cs_last_error_detail()
     assert call(L=0, nc=0) == cslib.CS_OK
