@@ -730,6 +730,38 @@ def cpu_baseline(w, x, layers, n_rows):
                               "full_step_s_est": round(t1[0]["full_step_s_est"], 3)}}
 
 
+def cpu_next_rows(w, k_l, v_l, n_rows: int, seed: int = 0) -> dict:
+    """The oracle's scatter-back and shallow-recompute attention on the host (one process),
+    on a bounded sample of the same work as `next_rows`, scaled to the full work:
+
+    * scatter_rows of the k repaired rows into one layer of K (seeded fresh rows at the step's
+      selected positions), scaled by 2 x L (K and V of every layer);
+    * repair_attention of n_rows seeded candidate rows at one layer, scaled by 2 layers x
+      sum(pos + 1) over all candidates / over the sampled ones.
+    k_l, v_l: fp64 [T, Hkv, D], one layer of the GPU arm's stored cache."""
+    import oracle as O
+    rng = np.random.default_rng(seed)
+    idx = np.sort(rng.choice(np.arange(w.cand0, w.cand0 + w.n_cand), w.k, replace=False))
+    rows = rng.standard_normal((1, w.k, w.hkv, w.head_dim))
+    t0 = time.perf_counter()
+    O.scatter_rows(k_l[None], rows, idx)
+    sc_s = (time.perf_counter() - t0) * 2 * w.n_layers
+    pos = np.arange(w.cand0, w.cand0 + w.n_cand, dtype=np.int64)
+    rsel = W.sample_rows(w.n_cand, n_rows, seed=seed + 1)
+    q = rng.standard_normal((1, len(rsel), w.hq, w.head_dim))
+    t0 = time.perf_counter()
+    O.repair_attention(q, k_l[None], v_l[None], pos[rsel].astype(np.int32))
+    nl = min(2, w.n_layers)
+    sr_s = (time.perf_counter() - t0) * nl * float(np.sum(pos + 1)) / float(np.sum(pos[rsel] + 1))
+    return {"cores": 1, "kind": "oracle", "value_is": "extrapolated from the sample",
+            "scatter_back": {"ms_est": round(sc_s * 1e3, 3),
+                             "sample": f"scatter_rows of {w.k} rows into 1 layer of K, x {2 * w.n_layers}"},
+            "shallow_recompute": {"ms_est": round(sr_s * 1e3, 1),
+                                  "sample": f"repair_attention of {len(rsel)} of {w.n_cand} "
+                                            f"candidate rows at 1 layer, x {nl} layers x "
+                                            "sum(pos+1) over all / over the sampled rows"}}
+
+
 def run_reference(args, w, ws):
     """The reference arm: the oracle (the paper publishes no code) on the host cores."""
     layers = [w.score_layer]
@@ -808,6 +840,10 @@ def main():
         xs = {"k": pristine[layers], "v": x["v"][layers], "q": x["q"][layers],
               "k_fresh_local": x["k_fresh_local"]}
         line["cpu_baseline"] = cpu_baseline(w, xs, layers, args.cpu_rows)
+        if "next_rows" in line:
+            f64 = lambda t: t.detach().float().cpu().numpy().astype(np.float64)   # noqa: E731
+            line["cpu_baseline"]["next_rows"] = cpu_next_rows(w, f64(xs["k"][0]), f64(xs["v"][0]),
+                                                              args.cpu_rows)
     if rank == 0:
         print(json.dumps(line), flush=True)
     if ws > 1:
