@@ -31,7 +31,9 @@ def test_pipeline_matches_oracle(cslib, name):
     # ---- oracle inputs: exact copies of the stored tensors, taken before the GPU runs
     k_score_layer = f64(x["k"][w.score_layer, cand])
     fresh_local = f64(x["k_fresh_local"])
-    layers = [0, w.n_layers - 1] if w.n_layers > 1 else [0]
+    # sampled layers: the first, the score layer, the quarters and the last
+    L = w.n_layers
+    layers = sorted({0, w.score_layer, L // 4, L // 2, (3 * L) // 4, L - 1})
     k_stored = {l: f64(x["k"][l]) for l in layers}
     # ---- GPU: fresh keys at global coordinates (the shallow recompute's output) ...
     fresh = torch.empty_like(x["k_fresh_local"])
@@ -57,7 +59,7 @@ def test_pipeline_matches_oracle(cslib, name):
     assert np.array_equal(got_qpos, exp_qpos), \
         f"{np.sum(got_qpos != exp_qpos)} selected indices differ"
     # attention over the composed cache, oracle fed its own re-based keys of the sampled layers
-    rows = W.sample_rows(w.M, 32 if w.T > 5000 else w.M, seed=9)
+    rows = W.sample_rows(w.M, 256 if w.T > 5000 else w.M, seed=9)
     for l in layers:
         k_l, _ = O.rebase(k_stored[l][None], loc, glo, dname)
         v_l = f64(x["v"][l])[None]
