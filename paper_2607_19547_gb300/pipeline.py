@@ -24,7 +24,10 @@ Options around the four calls:
   * GraphedQuery: a whole end-to-end query (input copies, the launches, output
     copies) captured once as a CUDA graph and replayed with one launch;
   * PipelinedQuery: the same with uploads, kernels and downloads overlapped layer
-    group by layer group on three streams (short first and last groups), also one graph.
+    group by layer group on three streams (short first and last groups), also one graph;
+  * QueryStream: a stream of such queries with several in flight (one PipelinedQuery
+    graph per slot, each slot on its own stream), so one query's uploads overlap
+    another's kernels and downloads.
 """
 from __future__ import annotations
 
@@ -252,6 +255,63 @@ class PipelinedQuery:
     def replay(self):
         """Runs the captured query (asynchronously, ordered after the current stream's work)."""
         self.graph.replay()
+        return self.h2d, self.d2h
+
+
+class QueryStream:
+    """A stream of end-to-end queries from host memory with n_slots queries in flight.
+
+    Each slot owns its device buffers (keys, values, queries and fresh keys; scores, query
+    positions and output through its own ComposedQuery), pinned host output buffers, a CUDA
+    stream and a captured PipelinedQuery graph.  Query i runs in slot i % n_slots on that
+    slot's stream, so a slot starts its next query only after its previous one, while the other
+    slots' queries overlap it: one query's uploads and first kernels run while another query
+    computes or downloads its result.  Every query still copies its own inputs in and its
+    result out.
+
+    host: the pinned host inputs (k, v, q, k_fresh), one dict shared by every slot or a list
+    with one dict per slot; pos_local, pos_global: device coordinates, shared read-only."""
+
+    def __init__(self, shape: QueryShape, dtype: torch.dtype, host, pos_local, pos_global,
+                 n_slots: int = 2, group_layers: int = 4, policy: str = "3axis"):
+        if n_slots < 1:
+            raise ValueError("n_slots must be at least 1")
+        hosts = list(host) if isinstance(host, (list, tuple)) else [host] * n_slots
+        if len(hosts) != n_slots:
+            raise ValueError("host must be one dict or one dict per slot")
+        self.device = pos_local.device
+        self.n_slots = n_slots
+        self.slots = []
+        for h in hosts:
+            q = ComposedQuery(shape, dtype, device=self.device)
+            dev = {n: torch.empty(h[n].shape, dtype=h[n].dtype, device=self.device)
+                   for n in ("k", "v", "q", "k_fresh")}
+            dev.update(pos_local=pos_local, pos_global=pos_global)
+            out_host = {"o": torch.empty(q.out.shape, dtype=q.out.dtype).pin_memory(),
+                        "qpos": torch.empty(shape.M, dtype=torch.int32).pin_memory()}
+            pq = PipelinedQuery(q, h, dev, out_host, group_layers=group_layers, policy=policy)
+            self.slots.append({"query": q, "dev": dev, "out_host": out_host, "graph": pq,
+                               "stream": torch.cuda.Stream(device=self.device)})
+        self.h2d = self.slots[0]["graph"].h2d
+        self.d2h = self.slots[0]["graph"].d2h
+
+    def out_host(self, slot: int) -> dict:
+        """The pinned host outputs (o, qpos) of `slot`: its last query's result."""
+        return self.slots[slot]["out_host"]
+
+    def run(self, n_queries: int):
+        """Launches n_queries queries, query i in slot i % n_slots, ordered after the current
+        stream's work; the current stream then waits for all of them (asynchronous to the
+        host).  Returns the bytes copied per query (host->device, device->host)."""
+        cur = torch.cuda.current_stream(self.device)
+        for s in self.slots:
+            s["stream"].wait_stream(cur)
+        for i in range(n_queries):
+            s = self.slots[i % self.n_slots]
+            with torch.cuda.stream(s["stream"]):
+                s["graph"].replay()
+        for s in self.slots:
+            cur.wait_stream(s["stream"])
         return self.h2d, self.d2h
 
 

@@ -100,3 +100,40 @@ def test_pipelined_query_equals_eager(cslib, name, policy, group, bounds):
             assert np.array_equal(bits16(got["o"]), bits16(eager["o"]))
         else:
             assert torch.equal(got["o"], eager["o"])
+
+
+@pytest.mark.parametrize("name", ["tiny_f32", "qwen3b_4x1024"])
+def test_query_stream_equals_eager(cslib, name):
+    """A stream of queries with two in flight: every slot's result equals the eager query on
+    that slot's host inputs, bit for bit, while the other slot's query overlaps it."""
+    from paper_2607_19547_gb300.pipeline import QueryStream
+    w = W.CONFIGS[name]
+    shape, host0, dev = _setup(w, 41)
+    # slot 1 serves other queries (new q rows) over the same cache
+    host1 = dict(host0)
+    host1["q"] = torch.randn(host0["q"].shape, generator=torch.Generator().manual_seed(5)).to(
+        host0["q"].dtype).pin_memory()
+    expect = []
+    for h in (host0, host1):
+        qe = ComposedQuery(shape, w.torch_dtype)
+        eo = _out_host(qe, w)
+        dev_e = {k: (v.clone() if k in ("k", "v", "q", "k_fresh") else v) for k, v in dev.items()}
+        compose_from_host(qe, h, dev_e, eo)
+        torch.cuda.synchronize()
+        expect.append(eo)
+    qs = QueryStream(shape, w.torch_dtype, [host0, host1], dev["pos_local"], dev["pos_global"],
+                     n_slots=2)
+    for n in (2, 5):
+        for s in range(2):
+            for t in qs.out_host(s).values():
+                t.zero_()
+        qs.run(n)
+        torch.cuda.synchronize()
+        cslib.cs_sync_status()
+        for s in range(2):
+            got, eo = qs.out_host(s), expect[s]
+            assert np.array_equal(got["qpos"].numpy(), eo["qpos"].numpy())
+            if w.dtype == "bf16":
+                assert np.array_equal(bits16(got["o"]), bits16(eo["o"]))
+            else:
+                assert torch.equal(got["o"], eo["o"])
