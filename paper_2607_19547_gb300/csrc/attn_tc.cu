@@ -23,15 +23,17 @@
 //   warps 2-9   softmax, two warpgroups: warpgroup h (warps 2+4h .. 5+4h)
 //               owns key columns [64h, 64h+64) of every S block and output
 //               dims [64h, 64h+64) of O; thread = one TMEM lane = one query
-//               row.  Reads its half of S_j, masks, takes the half-row maxima
-//               and computes its half of P_j = exp2(...) with the running max
-//               of the earlier blocks, then meets the warp that holds the
-//               other half of the same 32 rows (a 64-thread named barrier with
-//               an OR per block; the four row quarters run independently).
-//               The running max is raised only when it grows by more than
-//               2^8; when that happens in either half, both warps exchange
-//               their maxima through shared memory, raise it, recompute P_j
-//               from S_j and rescale their half of O in TMEM.  Each warp writes
+//               row.  Reads its half of S_j, masks it and computes its half of
+//               P_j = exp2(...) with the running max of the earlier blocks; the
+//               sum of those weights flags a block that may hold a larger
+//               maximum (above 2^12, or not finite).  It then meets the warp
+//               that holds the other half of the same 32 rows (a 64-thread
+//               named barrier with an OR per block; the four row quarters run
+//               independently).  When either half flagged (and on the first
+//               block), both warps take their half-row maxima of S_j, exchange
+//               them through shared memory, raise the running max if it grew by
+//               more than 2^8, recompute P_j from S_j and rescale their half of
+//               O in TMEM.  Each warp writes
 //               its half of P_j as bf16 over the first 32 of its own 64 S_j
 //               columns (never over columns the other warp reads), and the P*V
 //               issuer takes keys [64h, 64h+64) from columns [64h, 64h+32).
@@ -371,30 +373,19 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
             float psum = 0.0f;
             uint32_t pk[32];
             bool grow = true;   // the first block always sets the running max
-            if (ok) {
+            if (ok && j > 0) {
+                // this half of P_j with the running max of the earlier blocks; the sum of
+                // the weights flags a block that may hold a larger maximum (it exceeds 2^12,
+                // or is not finite), and only then do the warps take the half maxima (below)
                 tc_fence_after();
                 float s[64];
                 load_s_half(s_addr, diag, lim, s);
-                float mx4[4] = {s[0], s[1], s[2], s[3]};
-#pragma unroll
-                for (int c = 4; c < 64; c += 4) {
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) mx4[q] = fmaxf(mx4[q], s[c + q]);
-                }
-                const float mxh = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
-                slot[half * 128 + m] = mxh;
-                if (j > 0) {
-                    // this half of P_j with the running max of the earlier blocks, which
-                    // the row keeps unless its maximum grows by more than 2^8 in either
-                    // half (checked at the barrier below; then P_j is recomputed), so the
-                    // exponentials need not wait for the other half's maximum
-                    grow = mxh * p.scale_log2 > m_run + 8.0f;
-                    psum = exp_pack(s, p.scale_log2, m_run, pk);
-                }
+                psum = exp_pack(s, p.scale_log2, m_run, pk);
+                grow = !(psum <= 4096.0f);
             }
             // the two warps that own a row's halves (same TMEM lane quarter) meet here;
-            // the four pairs run independently of one another.  A failure or a raised
-            // maximum in either warp takes both through the exchange.
+            // the four pairs run independently of one another.  A failure or a flagged
+            // block in either warp takes both through the exchange of the half maxima.
             bool rescale = false;
             float alpha = 1.0f;
             if (named_bar_red_or(2 + qw, 64, !ok || grow)) {
@@ -403,6 +394,20 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
                     *abort = 1;
                     break;
                 }
+                // S_j is still in TMEM (P_j has not been written over it yet)
+                float s[64];
+                tc_fence_after();
+                load_s_half(s_addr, diag, lim, s);
+                {
+                    float mx4[4] = {s[0], s[1], s[2], s[3]};
+#pragma unroll
+                    for (int c = 4; c < 64; c += 4) {
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) mx4[q] = fmaxf(mx4[q], s[c + q]);
+                    }
+                    slot[half * 128 + m] = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
+                }
+                named_bar_sync(2 + qw, 64);   // both halves' maxima are in the slot
                 const float mx2 = fmaxf(slot[m], slot[128 + m]) * p.scale_log2;
                 const bool g = (m_run == -INFINITY) || (mx2 > m_run + 8.0f);
                 if (g) {
@@ -411,9 +416,6 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
                     m_run = mx2;
                 }
                 rescale = j > 0 && __any_sync(0xFFFFFFFFu, g);
-                // S_j is still in TMEM (P_j has not been written over it yet)
-                float s[64];
-                load_s_half(s_addr, diag, lim, s);
                 psum = exp_pack(s, p.scale_log2, m_run, pk);
             }
             // packed bf16 into columns [64h, 64h+32) of S_j's buffer: inside this warp's

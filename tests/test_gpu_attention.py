@@ -127,6 +127,25 @@ def test_bf16_max_grows_in_one_half(cslib):
                    qpos, "bf16")
 
 
+def test_bf16_growth_flag_thresholds(cslib):
+    """The regimes of the softmax's growth check (a block is flagged when its weights, taken with
+    the running maximum of the earlier blocks, sum above 2^12): one key about 2^10 above the
+    running maximum (not flagged: weights up to 2^10 stay in the running sum), then 64 keys of
+    one half block about 2^6.3 above it (flagged by their sum, while the maximum grows by less
+    than the 2^8 at which the running maximum is raised).  A constant query q = 0.5 against a
+    constant key c gives a log2-domain score of 0.5 * c * 128 / sqrt(128) * log2(e) = 8.16 c."""
+    L, T, Hq, Hkv = 1, 512, 8, 1
+    q = torch.full((L, 16, Hq, 128), 0.5, device="cuda")
+    k = _rand((L, T, Hkv, 128), 17, torch.float32) * 0.1
+    v = _rand((L, T, Hkv, 128), 18, torch.float32)
+    k[0, 150] = 10.0 / 8.16          # block 1, column 22: about 2^10 above block 0's maximum
+    k[0, 320:384] = 6.5 / 8.16       # block 2, columns 64-127: 64 weights of about 2^6.3
+    qpos = np.array([100, 149, 150, 151, 200, 255, 256, 300, 319, 320, 321, 350, 383, 384,
+                     450, 511], np.int32)
+    _run_and_check(cslib, q.to(torch.bfloat16), k.to(torch.bfloat16), v.to(torch.bfloat16),
+                   qpos, "bf16")
+
+
 def test_qwen3b_4x1024_all_rows(cslib):
     w = W.CONFIGS["qwen3b_4x1024"]
     x = W.make_inputs(w, seed=0, device="cuda")
