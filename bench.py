@@ -481,9 +481,10 @@ def run_gpu(args, w, ws, rank, local):
     pipe_mean = time_e2e(pipelined.replay)
     pipe_spread = spread[pipelined.replay]
     del pipelined, graphed
-    # a stream of queries with two in flight (one pipelined graph per slot, each slot with its
-    # own device buffers and stream): e2e_steps queries in one timed region, every query
-    # copying its own inputs in and its result out
+    # a stream of queries with two in flight (per slot: device buffers and captured graphs of
+    # the uploads, the launches and the downloads, on shared upload, compute and download
+    # streams): e2e_steps queries in one timed region, every query copying its own inputs in
+    # and its result out
     qstream = QueryStream(shape, w.torch_dtype, host, pl, pg, n_slots=2)
     qstream.run(2)
     torch.cuda.synchronize()
@@ -509,7 +510,8 @@ def run_gpu(args, w, ws, rank, local):
                    "steps": e2e_steps,
                    "h2d_gbs_effective": round(h2d / (e2e_mean / 1e3) / 1e9, 1),
                    "path": "QueryStream.run: the steps as a stream of queries, two in flight "
-                           "(one pipelined graph per slot on its own stream), one timed region",
+                           "(uploads, launches and downloads of each query as three graphs on "
+                           "shared upload, compute and download streams), one timed region",
                    "single_query": {
                        "value": round(replica_throughput(w.t_vis, pipe_mean, ws), 1),
                        "ms_per_step": round(pipe_mean, 4), "ms_min_median_max": pipe_spread,

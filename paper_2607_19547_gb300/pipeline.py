@@ -25,9 +25,10 @@ Options around the four calls:
     copies) captured once as a CUDA graph and replayed with one launch;
   * PipelinedQuery: the same with uploads, kernels and downloads overlapped layer
     group by layer group on three streams (short first and last groups), also one graph;
-  * QueryStream: a stream of such queries with several in flight (one PipelinedQuery
-    graph per slot, each slot on its own stream), so one query's uploads overlap
-    another's kernels and downloads.
+  * QueryStream: a stream of queries with several in flight (per slot, captured graphs of
+    the uploads, the launches and the downloads on shared upload, compute and download
+    streams), so one query's uploads and another's downloads overlap the computation
+    between them.
 """
 from __future__ import annotations
 
@@ -259,41 +260,72 @@ class PipelinedQuery:
 
 
 class QueryStream:
-    """A stream of end-to-end queries from host memory with n_slots queries in flight.
+    """A stream of end-to-end queries from host memory, n_slots of them in flight.
 
     Each slot owns its device buffers (keys, values, queries and fresh keys; scores, query
-    positions and output through its own ComposedQuery), pinned host output buffers, a CUDA
-    stream and a captured PipelinedQuery graph.  Query i runs in slot i % n_slots on that
-    slot's stream, so a slot starts its next query only after its previous one, while the other
-    slots' queries overlap it: one query's uploads and first kernels run while another query
-    computes or downloads its result.  Every query still copies its own inputs in and its
-    result out.
+    positions and output through its own ComposedQuery), pinned host output buffers, and three
+    captured CUDA graphs: the uploads of a query's inputs, its three launches, and the
+    downloads of its output and query positions.  Query i runs in slot i % n_slots: its
+    uploads go on the shared upload stream once the slot's previous query has finished
+    computing (its buffers are then free), its launches on the shared compute stream after its
+    uploads (and after the slot's previous download, which reads the output buffer), its
+    downloads on the shared download stream after its launches.  The queries' computations
+    thus run one after another while the next query's uploads and the previous query's
+    downloads overlap them: in steady state a query costs the longest of its upload, compute
+    and download times.  Every query copies its own inputs in and its result out.
 
     host: the pinned host inputs (k, v, q, k_fresh), one dict shared by every slot or a list
     with one dict per slot; pos_local, pos_global: device coordinates, shared read-only."""
 
     def __init__(self, shape: QueryShape, dtype: torch.dtype, host, pos_local, pos_global,
-                 n_slots: int = 2, group_layers: int = 4, policy: str = "3axis"):
+                 n_slots: int = 2, policy: str = "3axis"):
         if n_slots < 1:
             raise ValueError("n_slots must be at least 1")
+        if policy not in POLICIES:
+            raise ValueError(f"policy must be one of {POLICIES}")
         hosts = list(host) if isinstance(host, (list, tuple)) else [host] * n_slots
         if len(hosts) != n_slots:
             raise ValueError("host must be one dict or one dict per slot")
         self.device = pos_local.device
         self.n_slots = n_slots
+        self.s_up, self.s_c, self.s_down = (torch.cuda.Stream(device=self.device) for _ in range(3))
+        names = ("k", "v", "q", "k_fresh")
+        self.h2d = sum(hosts[0][n].numel() * hosts[0][n].element_size() for n in names)
         self.slots = []
+        side = torch.cuda.Stream(device=self.device)
+        side.wait_stream(torch.cuda.current_stream(self.device))
         for h in hosts:
             q = ComposedQuery(shape, dtype, device=self.device)
-            dev = {n: torch.empty(h[n].shape, dtype=h[n].dtype, device=self.device)
-                   for n in ("k", "v", "q", "k_fresh")}
-            dev.update(pos_local=pos_local, pos_global=pos_global)
+            dev = {n: torch.empty(h[n].shape, dtype=h[n].dtype, device=self.device) for n in names}
             out_host = {"o": torch.empty(q.out.shape, dtype=q.out.dtype).pin_memory(),
                         "qpos": torch.empty(shape.M, dtype=torch.int32).pin_memory()}
-            pq = PipelinedQuery(q, h, dev, out_host, group_layers=group_layers, policy=policy)
-            self.slots.append({"query": q, "dev": dev, "out_host": out_host, "graph": pq,
-                               "stream": torch.cuda.Stream(device=self.device)})
-        self.h2d = self.slots[0]["graph"].h2d
-        self.d2h = self.slots[0]["graph"].d2h
+
+            def upload(h=h, dev=dev):
+                for n in names:
+                    dev[n].copy_(h[n], non_blocking=True)
+
+            def compute(q=q, dev=dev):
+                q.step(dev["k"], dev["v"], dev["q"], dev["k_fresh"], pos_local, pos_global,
+                       stream=torch.cuda.current_stream(self.device), policy=policy)
+
+            def download(q=q, out_host=out_host):
+                out_host["o"].copy_(q.out, non_blocking=True)
+                out_host["qpos"].copy_(q.qpos, non_blocking=True)
+
+            graphs = []
+            with torch.cuda.stream(side):
+                for fn in (upload, compute, download):   # eager run: the library's set-up
+                    fn()
+            side.synchronize()
+            for fn in (upload, compute, download):
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g, stream=side):
+                    fn()
+                graphs.append(g)
+            self.slots.append({"query": q, "dev": dev, "out_host": out_host, "graphs": graphs,
+                               "ev": [torch.cuda.Event() for _ in range(3)], "used": False})
+        self.d2h = (self.slots[0]["query"].out.numel() * self.slots[0]["query"].out.element_size()
+                    + self.slots[0]["query"].qpos.numel() * 4)
 
     def out_host(self, slot: int) -> dict:
         """The pinned host outputs (o, qpos) of `slot`: its last query's result."""
@@ -304,14 +336,30 @@ class QueryStream:
         stream's work; the current stream then waits for all of them (asynchronous to the
         host).  Returns the bytes copied per query (host->device, device->host)."""
         cur = torch.cuda.current_stream(self.device)
-        for s in self.slots:
-            s["stream"].wait_stream(cur)
+        for st in (self.s_up, self.s_c, self.s_down):
+            st.wait_stream(cur)
         for i in range(n_queries):
             s = self.slots[i % self.n_slots]
-            with torch.cuda.stream(s["stream"]):
-                s["graph"].replay()
-        for s in self.slots:
-            cur.wait_stream(s["stream"])
+            g_up, g_c, g_down = s["graphs"]
+            ev_up, ev_c, ev_down = s["ev"]
+            if s["used"]:
+                self.s_up.wait_event(ev_c)      # the slot's previous query has read its inputs
+            with torch.cuda.stream(self.s_up):
+                g_up.replay()
+                ev_up.record(self.s_up)
+            self.s_c.wait_event(ev_up)
+            if s["used"]:
+                self.s_c.wait_event(ev_down)    # ... and its output has been downloaded
+            with torch.cuda.stream(self.s_c):
+                g_c.replay()
+                ev_c.record(self.s_c)
+            self.s_down.wait_event(ev_c)
+            with torch.cuda.stream(self.s_down):
+                g_down.replay()
+                ev_down.record(self.s_down)
+            s["used"] = True
+        for st in (self.s_up, self.s_c, self.s_down):
+            cur.wait_stream(st)
         return self.h2d, self.d2h
 
 
