@@ -68,3 +68,37 @@ def test_pipeline_matches_oracle(cslib, name):
         go = f64(out[l][torch.as_tensor(rows, device="cuda")])[None]
         err = np.max(np.abs(go - eo))
         assert err <= TOL[dname], f"layer {l}: max abs error {err}"
+
+
+def test_bench_workload_every_layer(cslib):
+    """The bench workload (64 chunks x 1024 tokens, rho 0.15) end to end, its attention checked
+    on every one of the 36 layers against the oracle run on that layer's own re-based keys, on 32
+    seeded rows (first and last included) per layer."""
+    w = W.CONFIGS["qwen3b_64x1024_r15"]
+    x = W.make_inputs(w, seed=3, device="cuda")
+    loc, glo = W.coordinates(w)
+    cand = slice(w.cand0, w.cand0 + w.n_cand)
+    k_stored = x["k"].clone()                     # the stored keys, before the in-place re-base
+    fresh = torch.empty_like(x["k_fresh_local"])
+    cslib.cs_rebase_keys(x["k_fresh_local"][None], cuda(loc[cand]), cuda(glo[cand]),
+                         k_out=fresh[None])
+    q = ComposedQuery(_shape(w), w.torch_dtype)
+    out, qpos = q.step(x["k"], x["v"], x["q"], fresh, cuda(loc), cuda(glo))
+    cslib.cs_sync_status()
+    # the selection, from the oracle's own re-base and score
+    kc_r, _ = O.rebase(f64(k_stored[w.score_layer, cand])[None], loc[cand], glo[cand], w.dtype)
+    kf_r, _ = O.rebase(f64(x["k_fresh_local"])[None], loc[cand], glo[cand], w.dtype)
+    score = O.score_f32_canonical(kf_r[0].astype(np.float32), kc_r[0].astype(np.float32))
+    exp_qpos = O.select_topk(score, w.k, w.cand0).astype(np.int32)
+    assert np.array_equal(qpos.cpu().numpy(), exp_qpos)
+    rows = W.sample_rows(w.M, 32, seed=13)
+    rows_dev = torch.as_tensor(rows, device="cuda")
+    worst = 0.0
+    for l in range(w.n_layers):
+        k_l, _ = O.rebase(f64(k_stored[l])[None], loc, glo, w.dtype)
+        eo, _ = O.repair_attention(f64(x["q"][l])[None][:, rows], k_l, f64(x["v"][l])[None],
+                                   exp_qpos[rows])
+        err = float(np.max(np.abs(f64(out[l][rows_dev])[None] - eo)))
+        worst = max(worst, err)
+        assert err <= TOL[w.dtype], f"layer {l}: max abs error {err}"
+    assert worst > 0.0          # the comparison ran on real values
