@@ -481,12 +481,14 @@ def run_gpu(args, w, ws, rank, local):
     pipe_mean = time_e2e(pipelined.replay)
     pipe_spread = spread[pipelined.replay]
     del pipelined, graphed
-    # a stream of queries with two in flight (per slot: device buffers and captured graphs of
-    # the uploads, the launches and the downloads, on shared upload, compute and download
-    # streams): e2e_steps queries in one timed region, every query copying its own inputs in
-    # and its result out
-    qstream = QueryStream(shape, w.torch_dtype, host, pl, pg, n_slots=2)
-    qstream.run(2)
+    # a stream of queries with up to four in flight (per slot: device buffers and captured
+    # graphs of the uploads, the launches and the downloads, on shared upload, compute and
+    # download streams; four slots let the uploads run up to three queries ahead, so a stall of
+    # the shared host link is absorbed): e2e_steps queries in one timed region, every query
+    # copying its own inputs in and its result out
+    n_slots = 4
+    qstream = QueryStream(shape, w.torch_dtype, host, pl, pg, n_slots=n_slots)
+    qstream.run(n_slots)
     torch.cuda.synchronize()
     flush_l2()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -509,7 +511,7 @@ def run_gpu(args, w, ws, rank, local):
                    "ms_per_step": round(e2e_mean, 4),
                    "steps": e2e_steps,
                    "h2d_gbs_effective": round(h2d / (e2e_mean / 1e3) / 1e9, 1),
-                   "path": "QueryStream.run: the steps as a stream of queries, two in flight "
+                   "path": f"QueryStream.run: the steps as a stream of queries, {n_slots} slots "
                            "(uploads, launches and downloads of each query as three graphs on "
                            "shared upload, compute and download streams), one timed region",
                    "single_query": {
