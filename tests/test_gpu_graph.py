@@ -102,35 +102,39 @@ def test_pipelined_query_equals_eager(cslib, name, policy, group, bounds):
             assert torch.equal(got["o"], eager["o"])
 
 
-@pytest.mark.parametrize("name", ["tiny_f32", "qwen3b_4x1024"])
-def test_query_stream_equals_eager(cslib, name):
-    """A stream of queries with two in flight: every slot's result equals the eager query on
-    that slot's host inputs, bit for bit, while the other slot's query overlaps it."""
+@pytest.mark.parametrize("name,n_slots", [("tiny_f32", 2), ("qwen3b_4x1024", 2),
+                                          ("qwen3b_4x1024", 4)])
+def test_query_stream_equals_eager(cslib, name, n_slots):
+    """A stream of queries with n_slots in flight: every slot's result equals the eager query on
+    that slot's host inputs, bit for bit, while the other slots' queries overlap it."""
     from paper_2607_19547_gb300.pipeline import QueryStream
     w = W.CONFIGS[name]
     shape, host0, dev = _setup(w, 41)
-    # slot 1 serves other queries (new q rows) over the same cache
-    host1 = dict(host0)
-    host1["q"] = torch.randn(host0["q"].shape, generator=torch.Generator().manual_seed(5)).to(
-        host0["q"].dtype).pin_memory()
+    # the other slots serve other queries (new q rows) over the same cache
+    hosts = [host0]
+    for s in range(1, n_slots):
+        h = dict(host0)
+        h["q"] = torch.randn(host0["q"].shape, generator=torch.Generator().manual_seed(5 + s)).to(
+            host0["q"].dtype).pin_memory()
+        hosts.append(h)
     expect = []
-    for h in (host0, host1):
+    for h in hosts:
         qe = ComposedQuery(shape, w.torch_dtype)
         eo = _out_host(qe, w)
         dev_e = {k: (v.clone() if k in ("k", "v", "q", "k_fresh") else v) for k, v in dev.items()}
         compose_from_host(qe, h, dev_e, eo)
         torch.cuda.synchronize()
         expect.append(eo)
-    qs = QueryStream(shape, w.torch_dtype, [host0, host1], dev["pos_local"], dev["pos_global"],
-                     n_slots=2)
-    for n in (2, 5):
-        for s in range(2):
+    qs = QueryStream(shape, w.torch_dtype, hosts, dev["pos_local"], dev["pos_global"],
+                     n_slots=n_slots)
+    for n in (n_slots, 2 * n_slots + 1):
+        for s in range(n_slots):
             for t in qs.out_host(s).values():
                 t.zero_()
         qs.run(n)
         torch.cuda.synchronize()
         cslib.cs_sync_status()
-        for s in range(2):
+        for s in range(n_slots):
             got, eo = qs.out_host(s), expect[s]
             assert np.array_equal(got["qpos"].numpy(), eo["qpos"].numpy())
             if w.dtype == "bf16":
