@@ -102,3 +102,36 @@ def test_bench_workload_every_layer(cslib):
         worst = max(worst, err)
         assert err <= TOL[w.dtype], f"layer {l}: max abs error {err}"
     assert worst > 0.0          # the comparison ran on real values
+
+
+@pytest.mark.parametrize("rho_bp", [0, 10000])
+@pytest.mark.parametrize("base", ["tiny_f32", "qwen3b_4x1024"])
+def test_pipeline_degenerate_rho(cslib, base, rho_bp):
+    """The method's two ends, end to end: rho = 0 repairs no token (only the text-suffix rows
+    query the cache), rho = 1 repairs every candidate.  Selection and attention against the
+    oracle on the same inputs."""
+    w = W.CONFIGS[base].with_(rho_bp=rho_bp, suffix=8, n_layers=min(3, W.CONFIGS[base].n_layers))
+    assert w.k == (0 if rho_bp == 0 else w.n_cand)
+    x = W.make_inputs(w, seed=17, device="cuda")
+    loc, glo = W.coordinates(w)
+    cand = slice(w.cand0, w.cand0 + w.n_cand)
+    k_stored = f64(x["k"])
+    fresh = torch.empty_like(x["k_fresh_local"])
+    cslib.cs_rebase_keys(x["k_fresh_local"][None], cuda(loc[cand]), cuda(glo[cand]),
+                         k_out=fresh[None])
+    q = ComposedQuery(_shape(w), w.torch_dtype)
+    out, qpos = q.step(x["k"], x["v"], x["q"], fresh, cuda(loc), cuda(glo))
+    cslib.cs_sync_status()
+    kc_r, _ = O.rebase(k_stored[w.score_layer, cand][None], loc[cand], glo[cand], w.dtype)
+    kf_r, _ = O.rebase(f64(x["k_fresh_local"])[None], loc[cand], glo[cand], w.dtype)
+    score = O.score_f32_canonical(kf_r[0].astype(np.float32), kc_r[0].astype(np.float32))
+    sel = O.select_topk(score, w.k, w.cand0)
+    exp_qpos = np.concatenate([sel, np.arange(w.T - w.suffix, w.T)]).astype(np.int32)
+    if rho_bp == 10000:
+        assert np.array_equal(sel, np.arange(w.cand0, w.cand0 + w.n_cand))
+    assert np.array_equal(qpos.cpu().numpy(), exp_qpos)
+    rows = W.sample_rows(w.M, 64, seed=19)
+    k_r, _ = O.rebase(k_stored, loc, glo, w.dtype)
+    eo, _ = O.repair_attention(f64(x["q"])[:, rows], k_r, f64(x["v"]), exp_qpos[rows])
+    go = f64(out[:, torch.as_tensor(rows, device="cuda")])
+    assert np.max(np.abs(go - eo)) <= TOL[w.dtype]
