@@ -482,10 +482,10 @@ def run_gpu(args, w, ws, rank, local):
     pipe_spread = spread[pipelined.replay]
     del pipelined, graphed
     # a stream of queries with up to four in flight (per slot: device buffers and captured
-    # graphs of the uploads, the launches and the downloads, on shared upload, compute and
-    # download streams; four slots let the uploads run up to three queries ahead, so a stall of
-    # the shared host link is absorbed): e2e_steps queries in one timed region, every query
-    # copying its own inputs in and its result out
+    # graphs of the uploads, the launches and the downloads of each layer part, on shared
+    # upload, compute and download streams; four slots let the uploads run up to three queries
+    # ahead, so a stall of the shared host link is absorbed): e2e_steps queries in one timed
+    # region, every query copying its own inputs in and its result out
     n_slots = 4
     qstream = QueryStream(shape, w.torch_dtype, host, pl, pg, n_slots=n_slots)
     qstream.run(n_slots)
@@ -512,8 +512,9 @@ def run_gpu(args, w, ws, rank, local):
                    "steps": e2e_steps,
                    "h2d_gbs_effective": round(h2d / (e2e_mean / 1e3) / 1e9, 1),
                    "path": f"QueryStream.run: the steps as a stream of queries, {n_slots} slots "
-                           "(uploads, launches and downloads of each query as three graphs on "
-                           "shared upload, compute and download streams), one timed region",
+                           "(uploads, launches and downloads of each layer part of a query as "
+                           "graphs on shared upload, compute and download streams), one timed "
+                           "region",
                    "single_query": {
                        "value": round(replica_throughput(w.t_vis, pipe_mean, ws), 1),
                        "ms_per_step": round(pipe_mean, 4), "ms_min_median_max": pipe_spread,

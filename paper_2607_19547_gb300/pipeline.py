@@ -149,6 +149,29 @@ class GraphedQuery:
         return self.h2d, self.d2h
 
 
+def _group_launches(q: ComposedQuery, dev: dict, a: int, b: int, policy: str, stream):
+    """The launches of one query for layers [a, b) on `stream`: re-base (for the group that
+    holds the score layer, with the score and the selection), then the repair attention of
+    those layers.  Every group's attention reads the selection, which the score layer's group
+    makes, so that group comes first in stream order."""
+    s = q.shape
+    k = dev["k"][a:b]
+    target = dev["pos_global"] if policy == "3axis" else q.scalar_targets()
+    if a <= s.score_layer < b:
+        if policy == "naive":
+            cached = dev["k"][s.score_layer, s.cand0:s.cand0 + s.n_cand]
+            cs_score_deviation(dev["k_fresh"], cached, out=q.score, stream=stream)
+        else:
+            cs_rebase_and_score(k, dev["pos_local"], target, dev["k_fresh"], s.score_layer - a,
+                                s.cand0, score_out=q.score, theta=s.theta, sections=s.sections,
+                                stream=stream)
+        cs_select_topk(q.score, s.k, s.cand0, out=q.qpos[:s.k], stream=stream)
+    elif policy != "naive":
+        cs_rebase_keys(k, dev["pos_local"], target, theta=s.theta, sections=s.sections,
+                       stream=stream)
+    cs_repair_attention(dev["q"][a:b], k, dev["v"][a:b], q.qpos, out=q.out[a:b], stream=stream)
+
+
 def plan_layer_groups(n_layers: int, score_layer: int, group_layers: int = 4, bounds=None):
     """Layer groups of a pipelined query, as (first, end) pairs covering [0, n_layers).
 
@@ -229,22 +252,7 @@ class PipelinedQuery:
                     dev[n][a:b].copy_(host[n][a:b], non_blocking=True)
             s_c.wait_stream(s_in)
             with torch.cuda.stream(s_c):
-                k = dev["k"][a:b]
-                target = dev["pos_global"] if policy == "3axis" else q.scalar_targets()
-                if a <= s.score_layer < b:
-                    if policy == "naive":
-                        cached = dev["k"][s.score_layer, s.cand0:s.cand0 + s.n_cand]
-                        cs_score_deviation(dev["k_fresh"], cached, out=q.score, stream=s_c)
-                    else:
-                        cs_rebase_and_score(k, dev["pos_local"], target, dev["k_fresh"],
-                                            s.score_layer - a, s.cand0, score_out=q.score,
-                                            theta=s.theta, sections=s.sections, stream=s_c)
-                    cs_select_topk(q.score, s.k, s.cand0, out=q.qpos[:s.k], stream=s_c)
-                elif policy != "naive":
-                    cs_rebase_keys(k, dev["pos_local"], target, theta=s.theta, sections=s.sections,
-                                   stream=s_c)
-                cs_repair_attention(dev["q"][a:b], k, dev["v"][a:b], q.qpos, out=q.out[a:b],
-                                    stream=s_c)
+                _group_launches(q, dev, a, b, policy, s_c)
             s_out.wait_stream(s_c)
             with torch.cuda.stream(s_out):
                 out_host["o"][a:b].copy_(q.out[a:b], non_blocking=True)
@@ -263,16 +271,18 @@ class QueryStream:
     """A stream of end-to-end queries from host memory, n_slots of them in flight.
 
     Each slot owns its device buffers (keys, values, queries and fresh keys; scores, query
-    positions and output through its own ComposedQuery), pinned host output buffers, and three
-    captured CUDA graphs: the uploads of a query's inputs, its three launches, and the
-    downloads of its output and query positions.  Query i runs in slot i % n_slots: its
-    uploads go on the shared upload stream once the slot's previous query has finished
-    computing (its buffers are then free), its launches on the shared compute stream after its
-    uploads (and after the slot's previous download, which reads the output buffer), its
-    downloads on the shared download stream after its launches.  The queries' computations
-    thus run one after another while the next query's uploads and the previous query's
-    downloads overlap them: in steady state a query costs the longest of its upload, compute
-    and download times.  Every query copies its own inputs in and its result out.
+    positions and output through its own ComposedQuery), pinned host output buffers, and, for
+    each of a query's layer parts (a short first part that holds the score layer, the middle,
+    a short last part), captured CUDA graphs of the part's uploads, launches and downloads.
+    Query i runs in slot i % n_slots: its uploads go on the shared upload stream once the
+    slot's previous query has finished computing (its buffers are then free), each part's
+    launches on the shared compute stream after that part's uploads (and after the slot's
+    previous download of the same part, which reads the output buffer), each part's download on
+    the shared download stream after its launches.  The queries' computations thus run one
+    after another while later queries upload and earlier ones download: in steady state a query
+    costs the longest of its upload, compute and download times, and the parts shorten what the
+    first query waits for its inputs and the last one for its output.  Every query copies its
+    own inputs in and its result out.
 
     host: the pinned host inputs (k, v, q, k_fresh), one dict shared by every slot or a list
     with one dict per slot; pos_local, pos_global: device coordinates, shared read-only."""
@@ -288,44 +298,56 @@ class QueryStream:
             raise ValueError("host must be one dict or one dict per slot")
         self.device = pos_local.device
         self.n_slots = n_slots
+        self.parts = plan_layer_groups(shape.n_layers, shape.score_layer,
+                                       group_layers=shape.n_layers)
         self.s_up, self.s_c, self.s_down = (torch.cuda.Stream(device=self.device) for _ in range(3))
         names = ("k", "v", "q", "k_fresh")
         self.h2d = sum(hosts[0][n].numel() * hosts[0][n].element_size() for n in names)
         self.slots = []
         side = torch.cuda.Stream(device=self.device)
         side.wait_stream(torch.cuda.current_stream(self.device))
+        last = len(self.parts) - 1
         for h in hosts:
             q = ComposedQuery(shape, dtype, device=self.device)
             dev = {n: torch.empty(h[n].shape, dtype=h[n].dtype, device=self.device) for n in names}
+            dev.update(pos_local=pos_local, pos_global=pos_global)
             out_host = {"o": torch.empty(q.out.shape, dtype=q.out.dtype).pin_memory(),
                         "qpos": torch.empty(shape.M, dtype=torch.int32).pin_memory()}
 
-            def upload(h=h, dev=dev):
-                for n in names:
-                    dev[n].copy_(h[n], non_blocking=True)
+            def upload(p, a, b, h=h, dev=dev):
+                if p == 0:
+                    dev["k_fresh"].copy_(h["k_fresh"], non_blocking=True)
+                for n in ("k", "v", "q"):
+                    dev[n][a:b].copy_(h[n][a:b], non_blocking=True)
 
-            def compute(q=q, dev=dev):
-                q.step(dev["k"], dev["v"], dev["q"], dev["k_fresh"], pos_local, pos_global,
-                       stream=torch.cuda.current_stream(self.device), policy=policy)
+            def compute(p, a, b, q=q, dev=dev):
+                _group_launches(q, dev, a, b, policy, torch.cuda.current_stream(self.device))
 
-            def download(q=q, out_host=out_host):
-                out_host["o"].copy_(q.out, non_blocking=True)
-                out_host["qpos"].copy_(q.qpos, non_blocking=True)
+            def download(p, a, b, q=q, out_host=out_host):
+                out_host["o"][a:b].copy_(q.out[a:b], non_blocking=True)
+                if p == last:
+                    out_host["qpos"].copy_(q.qpos, non_blocking=True)
 
-            graphs = []
-            with torch.cuda.stream(side):
-                for fn in (upload, compute, download):   # eager run: the library's set-up
-                    fn()
+            phases = (upload, compute, download)
+            with torch.cuda.stream(side):          # eager run: the library's one-time set-up
+                for p, (a, b) in enumerate(self.parts):
+                    for fn in phases:
+                        fn(p, a, b)
             side.synchronize()
-            for fn in (upload, compute, download):
-                g = torch.cuda.CUDAGraph()
-                with torch.cuda.graph(g, stream=side):
-                    fn()
-                graphs.append(g)
+            graphs = []
+            for p, (a, b) in enumerate(self.parts):
+                per_part = []
+                for fn in phases:
+                    g = torch.cuda.CUDAGraph()
+                    with torch.cuda.graph(g, stream=side):
+                        fn(p, a, b)
+                    per_part.append(g)
+                graphs.append(per_part)
             self.slots.append({"query": q, "dev": dev, "out_host": out_host, "graphs": graphs,
-                               "ev": [torch.cuda.Event() for _ in range(3)], "used": False})
-        self.d2h = (self.slots[0]["query"].out.numel() * self.slots[0]["query"].out.element_size()
-                    + self.slots[0]["query"].qpos.numel() * 4)
+                               "ev": [[torch.cuda.Event() for _ in range(3)] for _ in self.parts],
+                               "used": False})
+        q0 = self.slots[0]["query"]
+        self.d2h = q0.out.numel() * q0.out.element_size() + q0.qpos.numel() * 4
 
     def out_host(self, slot: int) -> dict:
         """The pinned host outputs (o, qpos) of `slot`: its last query's result."""
@@ -338,25 +360,28 @@ class QueryStream:
         cur = torch.cuda.current_stream(self.device)
         for st in (self.s_up, self.s_c, self.s_down):
             st.wait_stream(cur)
+        last = len(self.parts) - 1
         for i in range(n_queries):
             s = self.slots[i % self.n_slots]
-            g_up, g_c, g_down = s["graphs"]
-            ev_up, ev_c, ev_down = s["ev"]
             if s["used"]:
-                self.s_up.wait_event(ev_c)      # the slot's previous query has read its inputs
-            with torch.cuda.stream(self.s_up):
-                g_up.replay()
-                ev_up.record(self.s_up)
-            self.s_c.wait_event(ev_up)
-            if s["used"]:
-                self.s_c.wait_event(ev_down)    # ... and its output has been downloaded
-            with torch.cuda.stream(self.s_c):
-                g_c.replay()
-                ev_c.record(self.s_c)
-            self.s_down.wait_event(ev_c)
-            with torch.cuda.stream(self.s_down):
-                g_down.replay()
-                ev_down.record(self.s_down)
+                # the slot's previous query has read its inputs once its last part is computed
+                self.s_up.wait_event(s["ev"][last][1])
+            for p in range(len(self.parts)):
+                with torch.cuda.stream(self.s_up):
+                    s["graphs"][p][0].replay()
+                    s["ev"][p][0].record(self.s_up)
+            for p in range(len(self.parts)):
+                ev_up, ev_c, ev_down = s["ev"][p]
+                self.s_c.wait_event(ev_up)
+                if s["used"]:
+                    self.s_c.wait_event(ev_down)    # this part's previous output is downloaded
+                with torch.cuda.stream(self.s_c):
+                    s["graphs"][p][1].replay()
+                    ev_c.record(self.s_c)
+                self.s_down.wait_event(ev_c)
+                with torch.cuda.stream(self.s_down):
+                    s["graphs"][p][2].replay()
+                    ev_down.record(self.s_down)
             s["used"] = True
         for st in (self.s_up, self.s_c, self.s_down):
             cur.wait_stream(st)
