@@ -102,9 +102,12 @@ def test_pipelined_query_equals_eager(cslib, name, policy, group, bounds):
             assert torch.equal(got["o"], eager["o"])
 
 
-@pytest.mark.parametrize("name,n_slots", [("tiny_f32", 2), ("qwen3b_4x1024", 2),
-                                          ("qwen3b_4x1024", 4)])
-def test_query_stream_equals_eager(cslib, name, n_slots):
+@pytest.mark.parametrize("name,n_slots,policy", [("tiny_f32", 2, "3axis"),
+                                                 ("qwen3b_4x1024", 2, "3axis"),
+                                                 ("qwen3b_4x1024", 4, "3axis"),
+                                                 ("qwen3b_4x1024", 2, "scalar1d"),
+                                                 ("qwen3b_4x1024", 3, "naive")])
+def test_query_stream_equals_eager(cslib, name, n_slots, policy):
     """A stream of queries with n_slots in flight: every slot's result equals the eager query on
     that slot's host inputs, bit for bit, while the other slots' queries overlap it."""
     from paper_2607_19547_gb300.pipeline import QueryStream
@@ -122,11 +125,11 @@ def test_query_stream_equals_eager(cslib, name, n_slots):
         qe = ComposedQuery(shape, w.torch_dtype)
         eo = _out_host(qe, w)
         dev_e = {k: (v.clone() if k in ("k", "v", "q", "k_fresh") else v) for k, v in dev.items()}
-        compose_from_host(qe, h, dev_e, eo)
+        compose_from_host(qe, h, dev_e, eo, policy=policy)
         torch.cuda.synchronize()
         expect.append(eo)
     qs = QueryStream(shape, w.torch_dtype, hosts, dev["pos_local"], dev["pos_global"],
-                     n_slots=n_slots)
+                     n_slots=n_slots, policy=policy)
     for n in (n_slots, 2 * n_slots + 1):
         for s in range(n_slots):
             for t in qs.out_host(s).values():
